@@ -1,0 +1,454 @@
+"""Benchmark of the Log_bQuant inference hot path on GB300.
+
+Workload (one step): the decode step of a Llama-3.2-1B-shaped model at batch
+1 -- all 16 layers x 7 linears (q/o 2048x2048, k/v 512x2048, gate/up
+8192x2048, down 2048x8192), 4-bit Log_b codes with a per-layer base drawn
+from U[1.2, 2.0], Student-t(4)*0.02 weights with 0.1 % x20 outliers, bf16
+activations, fp32 outputs.  The 112 logq_linear calls of a step are captured
+once in a CUDA graph and replayed; the step's 486 MB of codes exceed L2, so no
+flush is needed between steps.
+
+metric: GEMV HBM GB/s at batch 1, counting the algorithmic bytes of every
+linear (packed codes + activations + outputs) per step.  The same run also
+measures the other rows of the path -- quantise (absmax + quantise + pack) of
+the whole model and the prefill GEMM on Llama-3.1-8B shapes (2048 tokens) --
+each with its own roofline, and times the fp64 oracle on the host cores.
+
+python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+N > 1 runs N independent replicas (one per GPU, launched by torchrun).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+from paper_2607_01127_gb300 import workloads  # noqa: E402
+
+METRIC = "Log_b 4-bit GEMV HBM GB/s (% of ~8 TB/s) at batch 1; prefill GEMM TFLOP/s"
+WORKLOAD = "llama-3.2-1b decode step: 16 layers x {q,k,v,o,gate,up,down} 4-bit Log_b GEMV, batch 1"
+CFG_SEED = 1
+PREFILL_TOKENS = 2048
+
+
+def peaks():
+    try:
+        return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json"))), "measured"
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+def model_layers():
+    """(layer, proj, N, K, seed) for every linear of the 1B-shaped model."""
+    out = []
+    for layer in range(workloads.LLAMA_1B_LAYERS):
+        for pi, name in enumerate(workloads.PROJ_NAMES):
+            N, K = workloads.LLAMA_1B_SHAPES[name]
+            out.append((layer, name, N, K, workloads.layer_seed(CFG_SEED, layer, pi)))
+    return out
+
+
+def linear_bytes(N, K, B=1, bits=4):
+    return N * K * bits // 8 + B * K * 2 + B * N * 4
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        sm, smax, reasons = [], 0.0, set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax = max(smax, float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": smax, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def traffic_for(kernel: str, source: str):
+    """DRAM bytes per launch from the committed ncu summary, or None when the
+    kernel source changed since those counters were taken."""
+    try:
+        t = json.load(open(os.path.join(ROOT, "profiles", "traffic.json")))[kernel]
+        digest = hashlib.sha256(open(os.path.join(ROOT, source), "rb").read()).hexdigest()[:16]
+        return t["bytes_per_launch"] if t.get("source_sha") == digest else None
+    except Exception:
+        return None
+
+
+# ----------------------------------------------------------------- oracle ---
+
+def oracle_gemv_sample(rows_per_layer: int = 8, seed: int = 0):
+    """Inputs of the CPU baseline: the first rows of every linear of the model,
+    quantised by the oracle (setup, untimed)."""
+    import oracle
+    bases = workloads.layer_bases(workloads.LLAMA_1B_LAYERS, CFG_SEED)
+    items = []
+    for layer, name, N, K, s in model_layers():
+        w = workloads.weights_np(rows_per_layer, K, s + seed, outliers=True)
+        cb = oracle.build_codebook(4, float(bases[layer]), float(np.abs(w).max()))
+        packed = oracle.pack(oracle.quantize_log(w, cb), 4)
+        x = workloads.activations_np(1, K, s).astype(np.float32)
+        items.append((cb, packed, x.astype(np.float64), rows_per_layer, K))
+    return items
+
+
+def oracle_gemv_run(items, threads: int):
+    import oracle
+    nbytes = 0
+    for cb, packed, x, R, K in items:
+        bs = np.zeros(R, np.int64)
+        ns = np.arange(R, dtype=np.int64)
+        oracle.linear_sampled(x, packed, 4, cb, oracle.TABLE_BF16, bs, ns, nthreads=threads)
+        nbytes += linear_bytes(R, K)
+    return nbytes
+
+
+def cpu_baseline(seconds: float = 12.0):
+    threads = len(os.sched_getaffinity(0))
+    items = oracle_gemv_sample()
+    oracle_gemv_run(items, threads)
+    t0, nbytes, reps = time.perf_counter(), 0, 0
+    while time.perf_counter() - t0 < seconds:
+        nbytes += oracle_gemv_run(items, threads)
+        reps += 1
+    dt = time.perf_counter() - t0
+    return {"value": round(nbytes / dt / 1e9, 4), "unit": "GB/s", "cores": threads, "kind": "oracle",
+            "sample": f"fp64 oracle GEMV over the first 8 rows of all 112 linears of the decode step, "
+                      f"{reps} passes in {dt:.1f} s"}
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    threads = len(os.sched_getaffinity(0))
+    items = oracle_gemv_sample()
+    for _ in range(args.warmup):
+        oracle_gemv_run(items, threads)
+    t0 = time.perf_counter()
+    nbytes = 0
+    for _ in range(args.steps):
+        nbytes += oracle_gemv_run(items, threads)
+    dt = time.perf_counter() - t0
+    v = nbytes / dt / 1e9
+    line = {"impl": "reference", "metric": METRIC, "value": round(v, 4), "unit": "GB/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(dt / args.steps * 1e3, 3), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD + " (oracle: first 8 rows of each linear per step)",
+                       "l2": "n/a (host)"},
+            "cpu_baseline": {"value": round(v, 4), "unit": "GB/s", "cores": threads, "kind": "oracle",
+                             "sample": "first 8 rows of each of the 112 linears per step"},
+            "e2e": {"value": round(v, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------- GPU arm ---
+
+def build_decode_model(logq, torch, dev):
+    bases = workloads.layer_bases(workloads.LLAMA_1B_LAYERS, CFG_SEED)
+    ws = logq.new_workspace(dev)
+    layers = []
+    for layer, name, N, K, s in model_layers():
+        W = workloads.weights_torch(N, K, s, outliers=True, device=dev)
+        codes, cb = logq.logq_quantize(W, 4, float(bases[layer]), workspace=ws)
+        del W
+        X = workloads.activations_torch(1, K, s, torch.bfloat16, dev)
+        Y = torch.empty(1, N, dtype=torch.float32, device=dev)
+        layers.append(dict(N=N, K=K, codes=codes, cb=cb, X=X, Y=Y, name=name))
+    return layers, ws
+
+
+def time_quantize(logq, torch, dev, reps: int = 2):
+    """Quantise every linear of the model (absmax pass + quantise-and-pack pass)."""
+    bases = workloads.layer_bases(workloads.LLAMA_1B_LAYERS, CFG_SEED)
+    ws = logq.new_workspace(dev)
+    shapes = [(layer, N, K, s) for layer, name, N, K, s in model_layers()][:7]  # one layer, all shapes
+    Ws = [workloads.weights_torch(N, K, s, outliers=True, device=dev) for _, N, K, s in shapes]
+    outs = [torch.empty(N * K // 2, dtype=torch.uint8, device=dev) for _, N, K, _ in shapes]
+    nweights = sum(N * K for _, N, K, _ in shapes)
+    for W, o, (layer, N, K, s) in zip(Ws, outs, shapes):
+        logq.logq_quantize(W, 4, float(bases[layer]), codes=o, workspace=ws)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(reps):
+        for W, o, (layer, N, K, s) in zip(Ws, outs, shapes):
+            logq.logq_quantize(W, 4, float(bases[layer]), codes=o, workspace=ws)
+    dt = (time.perf_counter() - t0) / reps          # logq_quantize synchronises per call
+    nbytes = nweights * (4 + 4 + 0.5)
+    return {"weights": nweights, "s": dt, "gbs": nbytes / dt / 1e9, "launches_per_pass": 2 * len(shapes),
+            "bytes_per_weight": 8.5}
+
+
+def time_prefill(logq, torch, dev, reps: int = 3):
+    """Prefill GEMM: 2048 tokens x each Llama-3.1-8B linear shape."""
+    res = {}
+    ws = logq.new_workspace(dev)
+    tot_flop, tot_t = 0.0, 0.0
+    for pi, name in enumerate(workloads.PROJ_NAMES):
+        if name in ("v", "up"):
+            continue                                 # same shapes as k and gate
+        N, K = workloads.LLAMA_8B_SHAPES[name]
+        W = workloads.weights_torch(N, K, workloads.layer_seed(4, 0, pi), outliers=True, device=dev)
+        codes, cb = logq.logq_quantize(W, 4, 1.5, workspace=ws)
+        del W
+        X = workloads.activations_torch(PREFILL_TOKENS, K, pi, torch.bfloat16, dev)
+        Y = torch.empty(PREFILL_TOKENS, N, dtype=torch.bfloat16, device=dev)
+        try:
+            logq.logq_linear(codes, cb, X, N, K, y_dtype=torch.bfloat16, Y=Y, workspace=ws)
+        except logq.LogqError as e:
+            if e.status == logq.LOGQ_ERR_UNSUPPORTED:
+                return None
+            raise
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            logq.logq_linear(codes, cb, X, N, K, y_dtype=torch.bfloat16, Y=Y, workspace=ws)
+        e1.record()
+        torch.cuda.synchronize()
+        t = e0.elapsed_time(e1) / reps * 1e-3
+        flop = 2.0 * PREFILL_TOKENS * N * K
+        res[name] = {"N": N, "K": K, "us": round(t * 1e6, 2), "tflops": round(flop / t / 1e12, 1)}
+        tot_flop += flop * (2 if name in ("k", "gate") else 1)
+        tot_t += t * (2 if name in ("k", "gate") else 1)
+        del codes, X, Y
+    st, _ = logq.logq_workspace_status(ws)
+    assert st == logq.LOGQ_OK, "prefill pipeline reported a timeout"
+    return {"layers": res, "tflops": tot_flop / tot_t / 1e12}
+
+
+def run_ours(args):
+    import torch
+    import paper_2607_01127_gb300 as logq
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    layers, ws = build_decode_model(logq, torch, dev)
+    step_bytes = sum(linear_bytes(L["N"], L["K"]) for L in layers)
+    launches_per_step = len(layers)
+    stream = torch.cuda.Stream(device=dev)
+
+    def step_calls():
+        for L in layers:
+            logq.logq_linear(L["codes"], L["cb"], L["X"], L["N"], L["K"], Y=L["Y"], workspace=ws,
+                             stream=stream)
+
+    with torch.cuda.stream(stream):
+        step_calls()                                          # warm-up outside capture
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(stream):
+        with torch.cuda.graph(graph, stream=stream):
+            step_calls()
+    for _ in range(args.warmup):
+        graph.replay()
+    barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clocks:
+        time.sleep(0.25)
+        barrier()
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(args.steps):
+                graph.replay()
+            e1.record(stream)
+        barrier()
+        time.sleep(0.25)
+    t = e0.elapsed_time(e1) * 1e-3
+    if dist is not None:
+        tt = torch.tensor([t], device=dev, dtype=torch.float64)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        t = float(tt.item())
+    value = step_bytes * args.steps * world / t / 1e9
+    ms_per_step = t / args.steps * 1e3
+
+    # e2e: activations from pinned host memory in, outputs to host out, every step
+    xh = torch.empty(sum(L["K"] for L in layers), dtype=torch.bfloat16, pin_memory=True)
+    yh = torch.empty(sum(L["N"] for L in layers), dtype=torch.float32, pin_memory=True)
+    xd = torch.empty_like(xh, device=dev)
+    off = 0
+    for L in layers:
+        xh[off:off + L["K"]].copy_(L["X"].view(-1).cpu())
+        L["Xv"] = xd[off:off + L["K"]].view(1, -1)
+        off += L["K"]
+    yd = torch.empty(yh.numel(), dtype=torch.float32, device=dev)
+    off = 0
+    for L in layers:
+        L["Yv"] = yd[off:off + L["N"]].view(1, -1)
+        off += L["N"]
+
+    def e2e_calls():
+        for L in layers:
+            logq.logq_linear(L["codes"], L["cb"], L["Xv"], L["N"], L["K"], Y=L["Yv"], workspace=ws,
+                             stream=stream)
+
+    g2 = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(stream):
+        e2e_calls()
+        torch.cuda.synchronize()
+        with torch.cuda.graph(g2, stream=stream):
+            e2e_calls()
+    h2d, d2h = xh.numel() * 2, yh.numel() * 4
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            xd.copy_(xh, non_blocking=True)
+            g2.replay()
+            yh.copy_(yd, non_blocking=True)
+        barrier()
+        f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        f0.record(stream)
+        for _ in range(args.steps):
+            xd.copy_(xh, non_blocking=True)
+            g2.replay()
+            yh.copy_(yd, non_blocking=True)
+        f1.record(stream)
+    barrier()
+    t2 = f0.elapsed_time(f1) * 1e-3
+    if dist is not None:
+        tt = torch.tensor([t2], device=dev, dtype=torch.float64)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        t2 = float(tt.item())
+    e2e_value = step_bytes * args.steps * world / t2 / 1e9
+    # the e2e output equals the device-resident run
+    assert torch.equal(yd[:layers[0]["N"]], layers[0]["Y"].view(-1))
+
+    pk, pk_kind = peaks()
+    gemv_bytes_per_launch = step_bytes / launches_per_step
+    achieved = gemv_bytes_per_launch / (t / args.steps / launches_per_step) / 1e9
+    tr = traffic_for("gemv_kernel", "paper_2607_01127_gb300/csrc/gemv.cu")
+    line = {
+        "metric": METRIC, "value": round(value, 1), "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": WORKLOAD, "global_batch": 1 * world, "linears_per_step": launches_per_step,
+                   "bytes_per_step": step_bytes, "bits": 4,
+                   "l2": "inputs larger than L2 (486 MB of codes per step vs 126 MB L2)",
+                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+                   "graph": "one CUDA graph per step, programmatic dependent launch between linears"},
+        "e2e": {"value": round(e2e_value, 1), "unit": "GB/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h},
+        "gpu_launches": launches_per_step * args.steps,
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": pk["hbm_gbs"], "unit": "GB/s",
+                     "frac": round(achieved / pk["hbm_gbs"], 4), "peak_source": pk_kind,
+                     "traffic": tr, "kernel": "gemv_kernel<4,1,32,8,bf16>",
+                     "algorithmic_bytes_per_launch": round(gemv_bytes_per_launch, 1),
+                     "frac_of_8TBs": round(achieved / 8000.0, 4)},
+        "clocks": clocks.summary(),
+    }
+    if rank == 0:
+        try:
+            q = time_quantize(logq, torch, dev)
+            line["quantize"] = {"gbs": round(q["gbs"], 1), "unit": "GB/s",
+                                "frac": round(q["gbs"] / pk["hbm_gbs"], 4),
+                                "weights_per_s": round(q["weights"] / q["s"], 1),
+                                "note": "absmax + quantise-and-pack of one layer's 7 linears, "
+                                        "8.5 B/weight algorithmic, host sync per call"}
+        except Exception as e:  # the headline line must still print
+            line["quantize"] = {"error": str(e)[:200]}
+        try:
+            pf = time_prefill(logq, torch, dev)
+            if pf is not None:
+                line["prefill"] = {"tflops": round(pf["tflops"], 1), "unit": "TFLOP/s",
+                                   "peak": pk["bf16_tflops"],
+                                   "frac": round(pf["tflops"] / pk["bf16_tflops"], 4),
+                                   "layers": pf["layers"], "tokens": PREFILL_TOKENS}
+            else:
+                line["prefill"] = None
+        except Exception as e:
+            line["prefill"] = {"error": str(e)[:200]}
+        if world == 1 and not args.no_cpu_baseline:
+            line["cpu_baseline"] = cpu_baseline()
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

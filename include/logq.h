@@ -1,0 +1,173 @@
+/*
+ * logq.h -- C ABI of the GB300 (sm_103a) Log_bQuant inference library.
+ *
+ * Log_bQuant stores each weight of a matrix as a sign + log-level code and
+ * decodes it through one codebook per matrix (paper Sec. 3.1):
+ *
+ *   Eq. (1)  Quant(b, s, x)   = 0 if x = 0, else sign(x) * round_clamp(log_b|x| + s)
+ *   Eq. (2)  Dequant(b, s, q) = 0 if q = 0, else sign(q) * b^(|q| - s)
+ *   q_max = 2^(n-1) - 1 for an n-bit code; Eq. (4) aligns w_max with q_max.
+ *
+ * Inference multiplies activations with the dequantised weights through a
+ * lookup table (Sec. 3.3).  This library provides the three steps of that
+ * path as device kernels behind plain C calls:
+ *   logq_build_codebook  host: (bits, base, range) -> levels and boundaries
+ *   logq_quantize        device: fp32 W[N][K] -> packed codes + codebook
+ *   logq_linear          device: codes, codebook, X[B][K] -> Y[B][N] = X * What^T
+ *
+ * Conventions shared by every call:
+ *   - Matrices are row-major and contiguous.  W and What are [N][K]
+ *     (PyTorch nn.Linear layout: out x in, K contiguous); X is [B][K];
+ *     Y is [B][N].
+ *   - "device" pointers are CUDA global-memory addresses on the current
+ *     device; "host" pointers are ordinary CPU memory.  The caller owns every
+ *     buffer; the library allocates no memory and keeps no per-call state.
+ *   - stream is a cudaStream_t passed as void*; NULL means the legacy default
+ *     stream.  Work is enqueued on that stream in order; calls return once it
+ *     is enqueued unless stated otherwise.
+ *   - Every argument is validated before anything is enqueued.  A call that
+ *     returns an error other than LOGQ_ERR_CUDA / LOGQ_ERR_NONFINITE has
+ *     touched no device memory.
+ *   - Device code never traps.  Conditions found on the device (non-finite
+ *     weights, a pipeline wait that exceeded its bound) are written to the
+ *     caller's workspace and reported by logq_quantize or logq_workspace_status.
+ */
+#ifndef LOGQ_H
+#define LOGQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    LOGQ_OK = 0,
+    LOGQ_ERR_INVALID_ARG = 1,   /* a size, pointer, alignment or parameter is invalid */
+    LOGQ_ERR_NONFINITE = 2,     /* W holds NaN or +-Inf */
+    LOGQ_ERR_UNSUPPORTED = 3,   /* valid request the library does not implement */
+    LOGQ_ERR_CUDA = 4,          /* a CUDA runtime call or launch failed */
+    LOGQ_ERR_WORKSPACE = 5,     /* workspace missing, too small or misaligned */
+    LOGQ_ERR_TIMEOUT = 6        /* a device-side pipeline wait hit its bound */
+} logq_status;
+
+typedef enum {
+    LOGQ_F32 = 0,
+    LOGQ_BF16 = 1,
+    LOGQ_F16 = 2
+} logq_dtype;
+
+/* flags of logq_build_codebook / logq_quantize */
+#define LOGQ_SHIFT_EXACT 0   /* s = q_max - log_b(range): the top level equals range (default) */
+#define LOGQ_SHIFT_FLOOR 1   /* s = q_max - floor(log_b range), Eq. (4) as printed */
+
+/*
+ * Codebook of one weight matrix (Sec. 3.1).  Plain data: the caller owns it
+ * and passes it by pointer; the library copies what it needs into kernel
+ * parameters.  Entries are indexed by the n-bit code c = sign << (n-1) | m:
+ *   level[m]               = +L_m,  level[2^(n-1) + m] = -L_m,
+ *   L_0 = 0 (level[2^(n-1)] = -0.0f), L_m = b^(m - s) for m = 1..q_max,
+ *   all rounded to nearest-even fp32 from an fp64 evaluation.
+ *   thresh[j] (j < q_max) is the decision boundary tau_j = b^(j + 1/2 - s)
+ *   between L_j and L_{j+1}, rounded UP to fp32, so that for an fp32 weight
+ *   |w| >= thresh[j] exactly when |w| >= tau_j.  Unused entries are +Inf.
+ *   level_bf16 / level_f16 are level[] rounded to nearest-even bf16 / fp16
+ *   (bit patterns); logq_linear multiplies with the table of X's dtype.
+ */
+typedef struct logq_codebook {
+    int32_t bits;            /* n: 3 or 4 */
+    int32_t qmax;            /* 2^(n-1) - 1 */
+    int32_t flags;           /* LOGQ_SHIFT_* used */
+    int32_t _pad;
+    double base;             /* b */
+    double shift;            /* s */
+    double range;            /* w_max the codebook was built for */
+    float level[16];
+    float thresh[8];
+    uint16_t level_bf16[16];
+    uint16_t level_f16[16];
+} logq_codebook;
+
+/*
+ * Packed code layout (produced by logq_quantize, consumed by logq_linear):
+ *   code of a weight: c = sign << (n-1) | m with m in 0..q_max and sign = 1
+ *   only for negative weights with m > 0.
+ *   n = 4: [N][K/2] bytes; byte j of a row holds k = 2j in bits 0-3 and
+ *          k = 2j+1 in bits 4-7.
+ *   n = 3: [N][3K/8] bytes; each run of 32 k is a 12-byte group of three
+ *          little-endian uint32 W0, W1, W2.  Pair p (k = 2p, 2p+1 of the group)
+ *          is the 6-bit field f_p = c(2p) | c(2p+1) << 3; for p = 5i + j
+ *          (i < 3, j < 5) f_p is bits [6j, 6j+6) of W_i; f_15 is split two
+ *          bits per word into bits 30-31 of W0 (f bits 0-1), W1 (2-3), W2 (4-5).
+ * K must be a positive multiple of 128 (rows stay 16-byte aligned).
+ */
+
+/* Fill *out for an n-bit codebook with base b = base > 1 and range > 0
+ * (Eq. (2) levels, Eq. (4) shift per flags).  Host only, no CUDA call.
+ * Errors: LOGQ_ERR_INVALID_ARG for bits not in {3,4}, base <= 1 or not
+ * finite, range <= 0 or not finite, unknown flags, out == NULL. */
+logq_status logq_build_codebook(int bits, double base, double range, int flags,
+                                logq_codebook* out);
+
+/* Bytes of packed codes for an N x K matrix at n bits (N*K/2 or N*3K/8);
+ * 0 when N <= 0, K is not a positive multiple of 128 or bits not in {3,4}. */
+size_t logq_packed_bytes(int64_t N, int64_t K, int bits);
+
+/* Bytes of device workspace that logq_quantize and logq_linear need (a small
+ * constant).  The caller allocates it (16-byte aligned), zero-fills it once,
+ * and may reuse it across calls on the same stream; calls that run at the
+ * same time on different streams need separate workspaces. */
+size_t logq_workspace_bytes(void);
+
+/*
+ * Quantise fp32 weights W[N][K] (device) to packed codes (device) with a
+ * codebook built for (bits, base, range, flags) -- Eq. (1) with the
+ * decision boundaries of logq_codebook: m = #{ j : |w| >= thresh[j] }.
+ *   range > 0: use it as w_max.  range <= 0: w_max = max|W| (Sec. 3.2),
+ *     computed on the device; one 8-byte device-to-host read follows.
+ *   cb_out (host, may be NULL) receives the codebook used.
+ *   codes must hold logq_packed_bytes(N, K, bits) bytes, 16-byte aligned;
+ *   W must be 16-byte aligned.
+ * Synchronises `stream` once before returning (to report non-finite weights).
+ * Errors: LOGQ_ERR_INVALID_ARG (sizes, pointers, alignment, codebook
+ * parameters), LOGQ_ERR_WORKSPACE, LOGQ_ERR_NONFINITE (W holds NaN/Inf; codes
+ * are then unspecified), LOGQ_ERR_CUDA. */
+logq_status logq_quantize(const float* W, int64_t N, int64_t K, int bits, double base,
+                          double range, int flags, uint8_t* codes, logq_codebook* cb_out,
+                          void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Y[B][N] = X[B][K] * What^T with What[n][k] = table[code(n, k)] (Sec. 3.3),
+ * accumulated in fp32.  table is cb->level_bf16 when x_dtype = LOGQ_BF16 and
+ * cb->level_f16 when x_dtype = LOGQ_F16.
+ *   codes (device): packed as above for cb->bits.  X (device): x_dtype.
+ *   Y (device): y_dtype in {LOGQ_F32, x_dtype}; a 16-bit Y is the fp32 sum
+ *   rounded to nearest-even.  All device pointers 16-byte aligned.
+ *   B <= 16 runs the decode GEMV / skinny-GEMM kernel on CUDA cores;
+ *   B > 16 runs the prefill GEMM kernel on the tensor cores (tcgen05).
+ * Asynchronous.  Errors: LOGQ_ERR_INVALID_ARG, LOGQ_ERR_UNSUPPORTED,
+ * LOGQ_ERR_WORKSPACE, LOGQ_ERR_CUDA (launch).  A device-side wait that hit
+ * its bound is reported later by logq_workspace_status. */
+logq_status logq_linear(const uint8_t* codes, const logq_codebook* cb, const void* X,
+                        logq_dtype x_dtype, int64_t B, int64_t N, int64_t K, void* Y,
+                        logq_dtype y_dtype, void* workspace, size_t workspace_bytes,
+                        void* stream);
+
+/* Synchronise `stream`, read the device error word of `workspace`, clear it,
+ * and return LOGQ_OK or LOGQ_ERR_TIMEOUT.  *detail (host, may be NULL)
+ * receives an implementation code naming the wait that gave up. */
+logq_status logq_workspace_status(void* workspace, void* stream, uint32_t* detail);
+
+/* Static description of a status code. */
+const char* logq_status_string(logq_status status);
+
+/* Number of streaming multiprocessors of the current device (0 on error);
+ * the persistent kernels size their grids from it. */
+int logq_device_sm_count(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LOGQ_H */

@@ -1,0 +1,494 @@
+// Decode GEMV / skinny GEMM on CUDA cores: Y[b][n] = sum_k X[b][k] * table[code(n, k)]
+// (paper Sec. 3.3: dequantisation by lookup table instead of exponentiation).
+//
+// Design (one persistent CTA of 16 warps per SM):
+//  * Pair table in shared memory.  Two codes (one byte at 4 bits, one 6-bit
+//    field at 3 bits) index a table whose entry is the bf16x2 / f16x2 pair of
+//    their dequantised values, signs included.  Each entry occupies a 256-byte
+//    row holding one copy per lane, so lane l always reads bank l: the lookups
+//    of a warp never conflict.  At 4 bits the byte offset of an entry,
+//    byte << 8 | 4 * lane, is one byte permute (prmt) of the code word.
+//  * Each warp owns a fixed span of K (32 lanes x KW consecutive k) and keeps
+//    its activations for that span in registers for the whole kernel; it walks
+//    the rows of the CTA's row range, one 16-, 8- or 4-byte coalesced load of
+//    codes per lane and row (a warp reads a contiguous 512/256/128-byte run).
+//  * fp32 accumulation (mixed-precision fma with bf16/f16 operands, or packed
+//    fp32 fma after unpacking), a reduce-scatter across the 32 lanes per round
+//    of rows, then a fixed-order sum over the spans in shared memory: results
+//    are bit-identical from run to run.
+//  * The CTA's contiguous range of code rows is prefetched into L2 with bulk
+//    prefetches at kernel start, so HBM streams at full rate while the warps
+//    consume from L2.
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <stdint.h>
+
+#include "internal.h"
+
+#ifndef LOGQ_GEMV_FMA_MODE
+#define LOGQ_GEMV_FMA_MODE 0   // 0: fma.rn.f32.{bf16,f16}; 1: fma.rn.f32x2 on unpacked bf16
+#endif
+
+namespace logq {
+namespace {
+
+constexpr int kThreads = 512;
+constexpr int kWarps = kThreads / 32;
+constexpr int kTabStride = 256;               // bytes per pair-table entry
+constexpr int kRedBytes = 60 * 1024;          // span-partial buffer
+constexpr int64_t kPrefetchCap = 1 << 20;     // bytes of codes prefetched per CTA up front
+// table (64 KiB at 4 bits) + up to 64 KiB of alignment pad + span partials
+constexpr int kMaxSmem = 65536 + 256 * kTabStride + kRedBytes;
+
+struct GemvParams {
+    const uint8_t* codes;
+    const uint16_t* X;
+    void* Y;
+    int64_t N;
+    int32_t K;
+    int32_t B;
+    int64_t row_bytes;
+    int32_t spans;        // S: spans of 32*KW k covering K
+    int32_t groups;       // G: warps sharing one span (row-parallel)
+    int32_t span_cols;    // warps / G: spans in flight at once
+    int32_t chunk_rows;   // rows reduced per shared-memory pass
+    int32_t y_dtype;
+    uint32_t lvl16[16];   // code-indexed 16-bit levels (low half used)
+};
+
+__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel)
+{
+    uint32_t r;
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(r) : "r"(a), "r"(b), "r"(sel));
+    return r;
+}
+
+__device__ __forceinline__ uint32_t lds32(uint32_t addr)
+{
+    uint32_t v;
+    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr));
+    return v;
+}
+
+template <int NW>
+struct CodeVec { uint32_t w[NW]; };
+
+template <int NW>
+__device__ __forceinline__ CodeVec<NW> ld_codes(const uint8_t* p)
+{
+    CodeVec<NW> c;
+    if constexpr (NW == 4) {
+        asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+                     : "=r"(c.w[0]), "=r"(c.w[1]), "=r"(c.w[2]), "=r"(c.w[3]) : "l"(p));
+    } else if constexpr (NW == 2) {
+        asm volatile("ld.global.nc.L1::no_allocate.v2.u32 {%0,%1}, [%2];"
+                     : "=r"(c.w[0]), "=r"(c.w[1]) : "l"(p));
+    } else {
+#pragma unroll
+        for (int i = 0; i < NW; ++i)
+            asm volatile("ld.global.nc.L1::no_allocate.u32 %0, [%1];" : "=r"(c.w[i]) : "l"(p + 4 * i));
+    }
+    return c;
+}
+
+template <bool F16>
+__device__ __forceinline__ void fma_pair(float& a0, float& a1, uint32_t w, uint32_t x)
+{
+#if LOGQ_GEMV_FMA_MODE == 0
+    if constexpr (F16) {
+        asm("{.reg .b16 wl, wh, xl, xh;\n\t"
+            "mov.b32 {wl, wh}, %2;\n\t"
+            "mov.b32 {xl, xh}, %3;\n\t"
+            "fma.rn.f32.f16 %0, wl, xl, %0;\n\t"
+            "fma.rn.f32.f16 %1, wh, xh, %1;}"
+            : "+f"(a0), "+f"(a1) : "r"(w), "r"(x));
+    } else {
+        asm("{.reg .b16 wl, wh, xl, xh;\n\t"
+            "mov.b32 {wl, wh}, %2;\n\t"
+            "mov.b32 {xl, xh}, %3;\n\t"
+            "fma.rn.f32.bf16 %0, wl, xl, %0;\n\t"
+            "fma.rn.f32.bf16 %1, wh, xh, %1;}"
+            : "+f"(a0), "+f"(a1) : "r"(w), "r"(x));
+    }
+#else
+    if constexpr (F16) {
+        asm("{.reg .b16 wl, wh, xl, xh;\n\t"
+            "mov.b32 {wl, wh}, %2;\n\t"
+            "mov.b32 {xl, xh}, %3;\n\t"
+            "fma.rn.f32.f16 %0, wl, xl, %0;\n\t"
+            "fma.rn.f32.f16 %1, wh, xh, %1;}"
+            : "+f"(a0), "+f"(a1) : "r"(w), "r"(x));
+    } else {
+        // bf16 -> fp32 is a 16-bit shift; x arrives unpacked the same way.
+        const float wl = __uint_as_float(w << 16), wh = __uint_as_float(w & 0xffff0000u);
+        const float xl = __uint_as_float(x << 16), xh = __uint_as_float(x & 0xffff0000u);
+        asm("{.reg .b64 a, b, c;\n\t"
+            "mov.b64 a, {%2, %3};\n\t"
+            "mov.b64 b, {%4, %5};\n\t"
+            "mov.b64 c, {%0, %1};\n\t"
+            "fma.rn.f32x2 c, a, b, c;\n\t"
+            "mov.b64 {%0, %1}, c;}"
+            : "+f"(a0), "+f"(a1) : "f"(wl), "f"(wh), "f"(xl), "f"(xh));
+    }
+#endif
+}
+
+// Reduce V per-lane values over the 32 lanes; afterwards lane l holds the
+// total of value index (l >> (5 - log2 V)) in a[0] (V <= 32, power of two).
+template <int V>
+__device__ __forceinline__ void reduce_scatter(float (&a)[V], int lane)
+{
+    int count = V;
+#pragma unroll
+    for (int m = 16; m >= 1; m >>= 1) {
+        if (count > 1) {
+            const int half = count / 2;
+            const bool upper = (lane & m) != 0;
+#pragma unroll
+            for (int i = 0; i < V / 2; ++i) {
+                if (i < half) {
+                    const float send = upper ? a[i] : a[i + half];
+                    const float keep = upper ? a[i + half] : a[i];
+                    a[i] = keep + __shfl_xor_sync(0xffffffffu, send, m);
+                }
+            }
+            count = half;
+        } else {
+            a[0] += __shfl_xor_sync(0xffffffffu, a[0], m);
+        }
+    }
+}
+
+__device__ __forceinline__ void store_y(void* Y, int dtype, int64_t idx, float v)
+{
+    if (dtype == LOGQ_F32) {
+        static_cast<float*>(Y)[idx] = v;
+    } else if (dtype == LOGQ_BF16) {
+        static_cast<__nv_bfloat16*>(Y)[idx] = __float2bfloat16_rn(v);
+    } else {
+        static_cast<__half*>(Y)[idx] = __float2half_rn(v);
+    }
+}
+
+// Shared-memory addresses of the four pair entries of one 4-bit code word.
+// base_lane holds 4 * lane in byte 0 and the table's 64 KiB-aligned shared
+// address in bytes 2-3, so one byte permute yields table + byte * 256 + 4 * lane.
+__device__ __forceinline__ void addrs4(uint32_t c, uint32_t base_lane, uint32_t (&o)[4])
+{
+    o[0] = prmt(c, base_lane, 0x7604u);
+    o[1] = prmt(c, base_lane, 0x7614u);
+    o[2] = prmt(c, base_lane, 0x7624u);
+    o[3] = prmt(c, base_lane, 0x7634u);
+}
+
+// Addresses of the 16 pair entries of one 3-bit group (W0, W1, W2); the
+// 6-bit field lands in bits 8-13, base_lane supplies the rest.
+__device__ __forceinline__ void addrs3(const uint32_t (&w)[3], uint32_t base_lane, uint32_t (&o)[16])
+{
+#pragma unroll
+    for (int i = 0; i < 3; ++i) {
+        o[5 * i + 0] = ((w[i] << 8) & 0x3f00u) | base_lane;
+        o[5 * i + 1] = ((w[i] << 2) & 0x3f00u) | base_lane;
+        o[5 * i + 2] = ((w[i] >> 4) & 0x3f00u) | base_lane;
+        o[5 * i + 3] = ((w[i] >> 10) & 0x3f00u) | base_lane;
+        o[5 * i + 4] = ((w[i] >> 16) & 0x3f00u) | base_lane;
+    }
+    o[15] = ((w[0] >> 22) & 0x0300u) | ((w[1] >> 20) & 0x0c00u) | ((w[2] >> 18) & 0x3000u) | base_lane;
+}
+
+// Decode one row's codes of this lane and accumulate B dot-product partials.
+template <int BITS, int B, int NW, bool F16, int NPAIR>
+__device__ __forceinline__ void decode_row(const CodeVec<NW>& c, uint32_t base_lane,
+                                           const uint32_t (&xr)[B][NPAIR], float* acc, float* acc_hi)
+{
+    if constexpr (BITS == 4) {
+#pragma unroll
+        for (int wi = 0; wi < NW; ++wi) {
+            uint32_t o[4];
+            addrs4(c.w[wi], base_lane, o);
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const uint32_t wp = lds32(o[j]);
+#pragma unroll
+                for (int b = 0; b < B; ++b) fma_pair<F16>(acc[b], acc_hi[b], wp, xr[b][4 * wi + j]);
+            }
+        }
+    } else {
+#pragma unroll
+        for (int gi = 0; gi < NW / 3; ++gi) {
+            uint32_t o[16];
+            const uint32_t w3[3] = {c.w[3 * gi], c.w[3 * gi + 1], c.w[3 * gi + 2]};
+            addrs3(w3, base_lane, o);
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                const uint32_t wp = lds32(o[j]);
+#pragma unroll
+                for (int b = 0; b < B; ++b) fma_pair<F16>(acc[b], acc_hi[b], wp, xr[b][16 * gi + j]);
+            }
+        }
+    }
+}
+
+template <int BITS, int B, int KW, int R, bool F16>
+__global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant__ GemvParams p)
+{
+    extern __shared__ __align__(16) uint8_t smem[];
+    constexpr int NPAIR = KW / 2;                            // bf16 pairs of x per lane and batch row
+    constexpr int NW = (BITS == 4) ? KW / 8 : 3 * KW / 32;   // code words per lane and row
+    constexpr int NENT = (BITS == 4) ? 256 : 64;
+    constexpr uint32_t TAB_BYTES = NENT * kTabStride;
+    constexpr int V = R * B;
+    constexpr int SPAN = 32 * KW;
+    static_assert(V <= 32 && (V & (V - 1)) == 0, "values per lane must be a power of two <= 32");
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int64_t C = gridDim.x;
+    const int64_t r0 = (p.N * (int64_t)blockIdx.x) / C;
+    const int64_t r1 = (p.N * ((int64_t)blockIdx.x + 1)) / C;
+
+    // 1) start streaming this CTA's code rows into L2.
+    {
+        const uint8_t* base = p.codes + r0 * p.row_bytes;
+        int64_t bytes = (r1 - r0) * p.row_bytes;
+        if (bytes > kPrefetchCap) bytes = kPrefetchCap;
+        constexpr int64_t piece = 16384;
+        for (int64_t off = (int64_t)tid * piece; off < bytes; off += (int64_t)kThreads * piece) {
+            const int64_t n = (bytes - off) < piece ? (bytes - off) : piece;
+            asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base + off), "r"((uint32_t)n)
+                         : "memory");
+        }
+    }
+
+    // 2) pair table at the first 64 KiB-aligned shared address of the
+    //    allocation; the span partials go below it when they fit, else above.
+    const uint32_t sbase = (uint32_t)__cvta_generic_to_shared(smem);
+    const uint32_t tab_addr = (sbase + 0xffffu) & ~0xffffu;
+    uint32_t* tab = reinterpret_cast<uint32_t*>(smem + (tab_addr - sbase));
+    const uint32_t red_bytes = (uint32_t)p.spans * (uint32_t)p.chunk_rows * B * 4u;
+    float* red = (tab_addr - sbase >= red_bytes) ? reinterpret_cast<float*>(smem)
+                                                 : reinterpret_cast<float*>(smem + (tab_addr - sbase) + TAB_BYTES);
+    // entry e = (value of its low code) | (value of its high code) << 16,
+    // 32 copies (one per lane) in the first 128 bytes of its 256-byte row.
+    for (int i = tid; i < NENT * 8; i += kThreads) {
+        const int e = i >> 3, part = i & 7;
+        const uint32_t lo = (BITS == 4) ? (e & 15) : (e & 7);
+        const uint32_t hi = (BITS == 4) ? (e >> 4) : (e >> 3);
+        const uint32_t v = (p.lvl16[lo] & 0xffffu) | (p.lvl16[hi] << 16);
+        reinterpret_cast<uint4*>(tab + e * (kTabStride / 4))[part] = make_uint4(v, v, v, v);
+    }
+    __syncthreads();
+    // 3) programmatic dependent launch: everything above touched only kernel
+    //    parameters, shared memory and an L2 hint, so it may overlap the tail of
+    //    the previous kernel on the stream.  X may be that kernel's output and Y
+    //    its input: wait for it before the first global read or write.
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+
+    const uint32_t base_lane = tab_addr | (4u * (uint32_t)lane);
+    const int G = p.groups, SC = p.span_cols;
+    const bool compute_warp = warp < G * SC;
+    const int g = warp % G, scol = warp / G;
+    constexpr int lg2V = (V >= 32) ? 5 : (V >= 16) ? 4 : (V >= 8) ? 3 : (V >= 4) ? 2 : (V >= 2) ? 1 : 0;
+    const int my_v = lane >> (5 - lg2V);
+    const bool writer = (lane & ((32 >> lg2V) - 1)) == 0;
+    const int64_t rstride = (int64_t)G * p.row_bytes;
+
+    for (int64_t q0 = r0; q0 < r1; q0 += p.chunk_rows) {
+        const int64_t q1 = (q0 + p.chunk_rows < r1) ? q0 + p.chunk_rows : r1;
+        const int nrows = (int)(q1 - q0);
+        const int my_rows = (nrows > g) ? (nrows - g + G - 1) / G : 0;
+        const int nrounds = (my_rows + R - 1) / R;
+        if (compute_warp && my_rows > 0) {
+            for (int s = scol; s < p.spans; s += SC) {
+                const int k0 = s * SPAN + lane * KW;
+                const bool active = k0 < p.K;
+                // activations for this span stay in registers (zero on idle lanes)
+                uint32_t xr[B][NPAIR];
+#pragma unroll
+                for (int b = 0; b < B; ++b) {
+                    const uint16_t* xp = p.X + (int64_t)b * p.K + (active ? k0 : 0);
+#pragma unroll
+                    for (int i = 0; i < NPAIR; i += 4) {
+                        uint4 v = make_uint4(0, 0, 0, 0);
+                        if (active && b < p.B) v = *reinterpret_cast<const uint4*>(xp + 2 * i);
+                        xr[b][i] = v.x;
+                        if (i + 1 < NPAIR) xr[b][i + 1] = v.y;
+                        if (i + 2 < NPAIR) xr[b][i + 2] = v.z;
+                        if (i + 3 < NPAIR) xr[b][i + 3] = v.w;
+                    }
+                }
+                // idle lanes read the row start (valid memory) and multiply by zero
+                const int64_t lane_byte = active ? ((BITS == 4) ? (int64_t)k0 / 2 : (int64_t)k0 / 32 * 12) : 0;
+                const uint8_t* first = p.codes + (q0 + g) * p.row_bytes + lane_byte;
+
+                // Rounds of R rows with two code buffers: the loads of round t+1 are
+                // in flight while round t is decoded.  Full rounds run unguarded;
+                // the last round guards its rows (warp-uniform branches).
+                CodeVec<NW> ca[R], cb[R];
+                auto load_round = [&](CodeVec<NW> (&c)[R], int t) {
+                    const int here = my_rows - t * R;
+                    const uint8_t* rp = first + (int64_t)t * R * rstride;
+#pragma unroll
+                    for (int r = 0; r < R; ++r)
+                        if (r < here) c[r] = ld_codes<NW>(rp + (int64_t)r * rstride);
+                };
+                auto run_round = [&](const CodeVec<NW> (&c)[R], int t) {
+                    const int here = my_rows - t * R;
+                    float acc[V], acc_hi[V];
+#pragma unroll
+                    for (int i = 0; i < V; ++i) acc[i] = acc_hi[i] = 0.f;
+                    if (here >= R) {
+#pragma unroll
+                        for (int r = 0; r < R; ++r) decode_row<BITS, B, NW, F16>(c[r], base_lane, xr, acc + r * B, acc_hi + r * B);
+                    } else {
+#pragma unroll
+                        for (int r = 0; r < R; ++r)
+                            if (r < here) decode_row<BITS, B, NW, F16>(c[r], base_lane, xr, acc + r * B, acc_hi + r * B);
+                    }
+#pragma unroll
+                    for (int i = 0; i < V; ++i) acc[i] += acc_hi[i];
+                    reduce_scatter<V>(acc, lane);
+                    if (writer) {
+                        const int r = my_v / B, b = my_v % B;
+                        const int lr = g + G * (t * R + r);
+                        if (lr < nrows) red[((int64_t)s * p.chunk_rows + lr) * B + b] = acc[0];
+                    }
+                };
+                load_round(ca, 0);
+                for (int t = 0; t < nrounds; t += 2) {
+                    if (t + 1 < nrounds) load_round(cb, t + 1);
+                    run_round(ca, t);
+                    if (t + 1 >= nrounds) break;
+                    if (t + 2 < nrounds) load_round(ca, t + 2);
+                    run_round(cb, t + 1);
+                }
+            }
+        }
+        __syncthreads();
+        // fixed-order sum over spans
+        for (int i = tid; i < nrows * B; i += kThreads) {
+            const int lr = i / B, b = i % B;
+            if (b >= p.B) continue;
+            float sum = 0.f;
+            for (int s = 0; s < p.spans; ++s) sum += red[((int64_t)s * p.chunk_rows + lr) * B + b];
+            store_y(p.Y, p.y_dtype, (int64_t)b * p.N + q0 + lr, sum);
+        }
+        __syncthreads();
+    }
+}
+
+struct Config {
+    int bits, B, KW, R;
+};
+
+// The dynamic shared-memory opt-in is a per-device function attribute: set it
+// once per device to the largest size any launch of this instantiation uses.
+template <int BITS, int B, int KW, int R, bool F16>
+cudaError_t run(const GemvParams& p, int grid, size_t smem, cudaStream_t s)
+{
+    auto k = gemv_kernel<BITS, B, KW, R, F16>;
+    static int configured[64] = {0};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    if (configured[dev] < (int)smem) {
+        e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem);
+        if (e != cudaSuccess) return e;
+        configured[dev] = kMaxSmem;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, k, p);
+}
+
+template <bool F16>
+cudaError_t dispatch(int bits, int Bp, const GemvParams& p, int grid, size_t smem, cudaStream_t s)
+{
+    if (bits == 4) {
+        switch (Bp) {
+        case 1: return run<4, 1, 32, 8, F16>(p, grid, smem, s);
+        case 2: return run<4, 2, 32, 4, F16>(p, grid, smem, s);
+        case 4: return run<4, 4, 16, 2, F16>(p, grid, smem, s);
+        case 8: return run<4, 8, 8, 1, F16>(p, grid, smem, s);
+        case 16: return run<4, 16, 8, 1, F16>(p, grid, smem, s);
+        }
+    } else {
+        switch (Bp) {
+        case 1: return run<3, 1, 32, 8, F16>(p, grid, smem, s);
+        case 2: return run<3, 2, 32, 4, F16>(p, grid, smem, s);
+        case 4: return run<3, 4, 32, 2, F16>(p, grid, smem, s);
+        }
+    }
+    return cudaErrorInvalidValue;
+}
+
+int padded_batch(int64_t B)
+{
+    if (B <= 1) return 1;
+    if (B <= 2) return 2;
+    if (B <= 4) return 4;
+    if (B <= 8) return 8;
+    return 16;
+}
+
+int kw_for(int bits, int Bp)
+{
+    if (bits == 3) return 32;
+    return Bp <= 2 ? 32 : (Bp == 4 ? 16 : 8);
+}
+
+}  // namespace
+
+bool gemv_supports(int bits, int64_t B)
+{
+    if (bits == 4) return B >= 1 && B <= 16;
+    if (bits == 3) return B >= 1 && B <= 4;
+    return false;
+}
+
+cudaError_t launch_gemv(const LinearArgs& a, cudaStream_t s)
+{
+    const int Bp = padded_batch(a.B);
+    const int KW = kw_for(a.bits, Bp);
+    const int span = 32 * KW;
+    GemvParams p;
+    p.codes = a.codes;
+    p.X = static_cast<const uint16_t*>(a.X);
+    p.Y = a.Y;
+    p.N = a.N;
+    p.K = (int32_t)a.K;
+    p.B = (int32_t)a.B;
+    p.row_bytes = (a.bits == 4) ? a.K / 2 : a.K / 32 * 12;
+    p.spans = (int32_t)((a.K + span - 1) / span);
+    if (p.spans >= kWarps) {
+        p.groups = 1;
+        p.span_cols = kWarps;
+    } else {
+        p.groups = kWarps / p.spans;
+        p.span_cols = p.spans;
+    }
+    const int sms = sm_count() > 0 ? sm_count() : 148;
+    const int64_t grid = a.N < sms ? a.N : sms;
+    const int64_t rows_per_cta = (a.N + grid - 1) / grid;
+    int64_t chunk = kRedBytes / ((int64_t)p.spans * Bp * 4);
+    if (chunk > rows_per_cta) chunk = rows_per_cta;
+    if (chunk < 1) return cudaErrorInvalidValue;
+    p.chunk_rows = (int32_t)chunk;
+    p.y_dtype = a.y_dtype;
+    for (int c = 0; c < 16; ++c) p.lvl16[c] = a.lvl16[c];
+    const int nent = (a.bits == 4) ? 256 : 64;
+    const size_t smem = 65536 + (size_t)nent * kTabStride + (size_t)p.spans * chunk * Bp * 4;
+    return a.x_f16 ? dispatch<true>(a.bits, Bp, p, (int)grid, smem, s)
+                   : dispatch<false>(a.bits, Bp, p, (int)grid, smem, s);
+}
+
+}  // namespace logq

@@ -1,0 +1,52 @@
+// Internal declarations shared by the translation units of liblogq.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "logq.h"
+
+namespace logq {
+
+// Workspace layout (logq_workspace_bytes() bytes, caller-allocated, zeroed once).
+struct Workspace {
+    uint32_t absmax_bits;   // max |w| as fp32 bits (atomicMax over non-negative floats)
+    uint32_t nonfinite;     // 1 when a NaN / Inf weight was seen
+    uint32_t error;         // device error word: LOGQ_ERR_TIMEOUT when a wait gave up
+    uint32_t detail;        // which wait gave up (implementation code)
+    uint32_t reserved[60];
+};
+static_assert(sizeof(Workspace) == 256, "workspace layout");
+constexpr size_t kWorkspaceBytes = sizeof(Workspace);
+
+// Decision boundaries handed to the quantise kernel (fp32, rounded up).
+struct QuantParams {
+    float thresh[8];
+    int32_t qmax;
+    int32_t bits;
+    int32_t check_nonfinite;
+    int32_t _pad;
+};
+
+// One quantised linear call after validation.
+struct LinearArgs {
+    const uint8_t* codes;
+    const void* X;
+    void* Y;
+    int64_t B, N, K;
+    int bits;
+    int x_f16;              // 0: bf16 activations, 1: fp16
+    int y_dtype;            // logq_dtype of Y
+    uint16_t lvl16[16];     // code-indexed 16-bit levels in X's dtype
+    Workspace* ws;
+};
+
+int sm_count();
+cudaError_t launch_absmax(const float* W, int64_t count, Workspace* ws, cudaStream_t s);
+cudaError_t launch_quantize(const float* W, int64_t N, int64_t K, const QuantParams& p,
+                            uint8_t* codes, Workspace* ws, cudaStream_t s);
+cudaError_t launch_gemv(const LinearArgs& a, cudaStream_t s);
+cudaError_t launch_prefill(const LinearArgs& a, cudaStream_t s);
+bool gemv_supports(int bits, int64_t B);
+
+}  // namespace logq

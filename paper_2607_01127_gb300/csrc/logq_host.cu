@@ -1,0 +1,266 @@
+// C-ABI front of liblogq: argument validation, the host codebook builder
+// (paper Sec. 3.1, Eqs. (2) and (4)) and dispatch to the device kernels.
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <math.h>
+#include <string.h>
+
+#include <mutex>
+
+#include "internal.h"
+
+namespace logq {
+
+int sm_count()
+{
+    static int cached[64] = {0};
+    static std::mutex mu;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+    std::lock_guard<std::mutex> g(mu);
+    if (cached[dev] == 0) {
+        int v = 0;
+        if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+        cached[dev] = v;
+    }
+    return cached[dev];
+}
+
+}  // namespace logq
+
+using namespace logq;
+
+namespace {
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Largest integer e with b^e <= x (x > 0, b > 1), settled with exact power
+// comparisons so that exact powers of b are not lost to rounding of log().
+long floor_log_base(double x, double b)
+{
+    long e = (long)floor(log(x) / log(b));
+    while (pow(b, (double)(e + 1)) <= x) ++e;
+    while (pow(b, (double)e) > x) --e;
+    return e;
+}
+
+// Smallest fp32 >= t for t > 0.
+float round_up_f32(double t)
+{
+    float f = (float)t;
+    while ((double)f < t) f = nextafterf(f, INFINITY);
+    for (;;) {
+        float g = nextafterf(f, 0.0f);
+        if ((double)g >= t) f = g;
+        else break;
+    }
+    return f;
+}
+
+uint16_t bf16_bits_of(float v)
+{
+    __nv_bfloat16 h = __float2bfloat16_rn(v);
+    uint16_t b;
+    memcpy(&b, &h, 2);
+    return b;
+}
+
+uint16_t f16_bits_of(float v)
+{
+    __half h = __float2half_rn(v);
+    uint16_t b;
+    memcpy(&b, &h, 2);
+    return b;
+}
+
+logq_status cuda_status(cudaError_t e) { return e == cudaSuccess ? LOGQ_OK : LOGQ_ERR_CUDA; }
+
+}  // namespace
+
+extern "C" {
+
+logq_status logq_build_codebook(int bits, double base, double range, int flags, logq_codebook* out)
+{
+    if (!out || (bits != 3 && bits != 4)) return LOGQ_ERR_INVALID_ARG;
+    if (!isfinite(base) || !(base > 1.0) || !isfinite(range) || !(range > 0.0))
+        return LOGQ_ERR_INVALID_ARG;
+    if (flags != LOGQ_SHIFT_EXACT && flags != LOGQ_SHIFT_FLOOR) return LOGQ_ERR_INVALID_ARG;
+
+    logq_codebook cb;
+    memset(&cb, 0, sizeof cb);
+    const int qmax = (1 << (bits - 1)) - 1;
+    cb.bits = bits;
+    cb.qmax = qmax;
+    cb.flags = flags;
+    cb.base = base;
+    cb.range = range;
+    // Eq. (4): s aligns w_max with q_max.  Exact mode keeps log_b(range)
+    // unrounded so the top level is the range itself; floor mode is Eq. (4)
+    // as printed.
+    const long e_floor = (flags == LOGQ_SHIFT_FLOOR) ? floor_log_base(range, base) : 0;
+    cb.shift = (flags == LOGQ_SHIFT_FLOOR) ? (double)qmax - (double)e_floor
+                                           : (double)qmax - log(range) / log(base);
+
+    // Eq. (2): L_m = b^(m - s).  Exact mode: b^(m - q_max) * range.
+    double L[8] = {0};
+    for (int m = 1; m <= qmax; ++m)
+        L[m] = (flags == LOGQ_SHIFT_FLOOR) ? pow(base, (double)m - cb.shift)
+                                           : range * pow(base, (double)(m - qmax));
+    const int half = 1 << (bits - 1);
+    for (int c = 0; c < 2 * half; ++c) {
+        const int m = c & (half - 1);
+        const float mag = (float)L[m];
+        const float v = (c & half) ? -mag : mag;
+        cb.level[c] = v;
+        cb.level_bf16[c] = bf16_bits_of(v);
+        cb.level_f16[c] = f16_bits_of(v);
+    }
+    // Decision boundary between L_j and L_{j+1}: round(log_b|w| + s) >= j + 1
+    // exactly when |w| >= b^(j + 1/2 - s).
+    for (int j = 0; j < 8; ++j) {
+        if (j < qmax) {
+            const double t = (flags == LOGQ_SHIFT_FLOOR)
+                                 ? pow(base, (double)j + 0.5 - cb.shift)
+                                 : range * pow(base, (double)j + 0.5 - (double)qmax);
+            cb.thresh[j] = round_up_f32(t);
+        } else {
+            cb.thresh[j] = INFINITY;
+        }
+    }
+    *out = cb;
+    return LOGQ_OK;
+}
+
+size_t logq_packed_bytes(int64_t N, int64_t K, int bits)
+{
+    if (N <= 0 || K <= 0 || (K % 128) != 0) return 0;
+    if (bits == 4) return (size_t)N * (size_t)(K / 2);
+    if (bits == 3) return (size_t)N * (size_t)(K / 32 * 12);
+    return 0;
+}
+
+size_t logq_workspace_bytes(void) { return kWorkspaceBytes; }
+
+logq_status logq_quantize(const float* W, int64_t N, int64_t K, int bits, double base,
+                          double range, int flags, uint8_t* codes, logq_codebook* cb_out,
+                          void* workspace, size_t workspace_bytes, void* stream)
+{
+    if (!W || !codes || !aligned16(W) || !aligned16(codes)) return LOGQ_ERR_INVALID_ARG;
+    if (logq_packed_bytes(N, K, bits) == 0) return LOGQ_ERR_INVALID_ARG;
+    if (!isfinite(base) || !(base > 1.0) || isnan(range) || isinf(range)) return LOGQ_ERR_INVALID_ARG;
+    if (flags != LOGQ_SHIFT_EXACT && flags != LOGQ_SHIFT_FLOOR) return LOGQ_ERR_INVALID_ARG;
+    if (!workspace || !aligned16(workspace) || workspace_bytes < kWorkspaceBytes)
+        return LOGQ_ERR_WORKSPACE;
+    if (N > (int64_t(1) << 40) / K) return LOGQ_ERR_INVALID_ARG;
+
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    Workspace* ws = static_cast<Workspace*>(workspace);
+    cudaError_t e = cudaMemsetAsync(ws, 0, 2 * sizeof(uint32_t), s);
+    if (e != cudaSuccess) return LOGQ_ERR_CUDA;
+
+    uint32_t host_words[2] = {0, 0};
+    const bool auto_range = !(range > 0.0);
+    if (auto_range) {
+        // Sec. 3.2: w_max = max_i |w_i|, reduced on the device.
+        if ((e = launch_absmax(W, N * K, ws, s)) != cudaSuccess) return LOGQ_ERR_CUDA;
+        if ((e = cudaMemcpyAsync(host_words, ws, sizeof host_words, cudaMemcpyDeviceToHost, s)) != cudaSuccess)
+            return LOGQ_ERR_CUDA;
+        if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return LOGQ_ERR_CUDA;
+        if (host_words[1]) return LOGQ_ERR_NONFINITE;
+        float mx;
+        memcpy(&mx, &host_words[0], 4);
+        if (!(mx > 0.0f)) return LOGQ_ERR_INVALID_ARG;   // all-zero weights: no log range
+        range = (double)mx;
+    }
+
+    logq_codebook cb;
+    logq_status st = logq_build_codebook(bits, base, range, flags, &cb);
+    if (st != LOGQ_OK) return st;
+
+    QuantParams p;
+    memset(&p, 0, sizeof p);
+    for (int j = 0; j < 8; ++j) p.thresh[j] = cb.thresh[j];
+    p.qmax = cb.qmax;
+    p.bits = bits;
+    p.check_nonfinite = auto_range ? 0 : 1;
+    if ((e = launch_quantize(W, N, K, p, codes, ws, s)) != cudaSuccess) return LOGQ_ERR_CUDA;
+    if (!auto_range) {
+        if ((e = cudaMemcpyAsync(host_words, ws, sizeof host_words, cudaMemcpyDeviceToHost, s)) != cudaSuccess)
+            return LOGQ_ERR_CUDA;
+        if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return LOGQ_ERR_CUDA;
+        if (host_words[1]) return LOGQ_ERR_NONFINITE;
+    } else {
+        if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return LOGQ_ERR_CUDA;
+    }
+    if (cb_out) *cb_out = cb;
+    return LOGQ_OK;
+}
+
+logq_status logq_linear(const uint8_t* codes, const logq_codebook* cb, const void* X,
+                        logq_dtype x_dtype, int64_t B, int64_t N, int64_t K, void* Y,
+                        logq_dtype y_dtype, void* workspace, size_t workspace_bytes, void* stream)
+{
+    if (!codes || !cb || !X || !Y) return LOGQ_ERR_INVALID_ARG;
+    if (!aligned16(codes) || !aligned16(X) || !aligned16(Y)) return LOGQ_ERR_INVALID_ARG;
+    if (B <= 0 || logq_packed_bytes(N, K, cb->bits) == 0) return LOGQ_ERR_INVALID_ARG;
+    if (cb->qmax != (1 << (cb->bits - 1)) - 1) return LOGQ_ERR_INVALID_ARG;
+    if (x_dtype != LOGQ_BF16 && x_dtype != LOGQ_F16) return LOGQ_ERR_UNSUPPORTED;
+    if (y_dtype != LOGQ_F32 && y_dtype != x_dtype) return LOGQ_ERR_UNSUPPORTED;
+    if (N > (int64_t(1) << 31) || K > (int64_t(1) << 30) || B > (int64_t(1) << 31))
+        return LOGQ_ERR_INVALID_ARG;
+    if (!workspace || !aligned16(workspace) || workspace_bytes < kWorkspaceBytes)
+        return LOGQ_ERR_WORKSPACE;
+
+    LinearArgs a;
+    memset(&a, 0, sizeof a);
+    a.codes = codes;
+    a.X = X;
+    a.Y = Y;
+    a.B = B;
+    a.N = N;
+    a.K = K;
+    a.bits = cb->bits;
+    a.x_f16 = (x_dtype == LOGQ_F16);
+    a.y_dtype = (int)y_dtype;
+    const uint16_t* tab = a.x_f16 ? cb->level_f16 : cb->level_bf16;
+    for (int c = 0; c < (1 << cb->bits); ++c) a.lvl16[c] = tab[c];
+    a.ws = static_cast<Workspace*>(workspace);
+
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (gemv_supports(cb->bits, B)) return cuda_status(launch_gemv(a, s));
+    const cudaError_t e = launch_prefill(a, s);
+    if (e == cudaErrorNotSupported) return LOGQ_ERR_UNSUPPORTED;
+    return cuda_status(e);
+}
+
+logq_status logq_workspace_status(void* workspace, void* stream, uint32_t* detail)
+{
+    if (!workspace || !aligned16(workspace)) return LOGQ_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    Workspace* ws = static_cast<Workspace*>(workspace);
+    uint32_t words[2] = {0, 0};
+    if (cudaMemcpyAsync(words, &ws->error, sizeof words, cudaMemcpyDeviceToHost, s) != cudaSuccess)
+        return LOGQ_ERR_CUDA;
+    if (cudaMemsetAsync(&ws->error, 0, sizeof words, s) != cudaSuccess) return LOGQ_ERR_CUDA;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return LOGQ_ERR_CUDA;
+    if (detail) *detail = words[1];
+    return words[0] ? LOGQ_ERR_TIMEOUT : LOGQ_OK;
+}
+
+const char* logq_status_string(logq_status status)
+{
+    switch (status) {
+    case LOGQ_OK: return "ok";
+    case LOGQ_ERR_INVALID_ARG: return "invalid argument";
+    case LOGQ_ERR_NONFINITE: return "weights contain NaN or Inf";
+    case LOGQ_ERR_UNSUPPORTED: return "unsupported configuration";
+    case LOGQ_ERR_CUDA: return "CUDA runtime error";
+    case LOGQ_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+    case LOGQ_ERR_TIMEOUT: return "device pipeline wait exceeded its bound";
+    }
+    return "unknown status";
+}
+
+int logq_device_sm_count(void) { return sm_count(); }
+
+}  // extern "C"

@@ -1,0 +1,162 @@
+"""Host-side tests of the C ABI (no GPU needed): the library builds and loads,
+exports every symbol that include/logq.h declares, builds the same codebooks
+as the oracle, sizes buffers, and rejects invalid arguments before touching
+the device."""
+import ctypes
+import math
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="session")
+def logq():
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2607_01127_gb300 as m
+    return m
+
+
+def declared_symbols():
+    src = open(os.path.join(ROOT, "include", "logq.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(logq_[a-z0-9_]+)\s*\(", src)))
+
+
+def test_exports_every_declared_symbol(logq):
+    names = declared_symbols()
+    assert len(names) >= 8
+    for n in names:
+        assert hasattr(logq.lib, n), n          # dlsym succeeds
+    assert set(names) == set(logq.EXPORTED)
+
+
+def test_struct_layout_matches_header(logq):
+    # 4 int32 + 3 double + 16 float + 8 float + 2 x 16 uint16
+    assert ctypes.sizeof(logq.Codebook) == 16 + 24 + 64 + 32 + 64
+
+
+@pytest.mark.parametrize("bits", [3, 4])
+@pytest.mark.parametrize("base", [1.2, 1.25, 1.5, 1.7351, 2.0])
+@pytest.mark.parametrize("rng_", [0.0173, 0.31, 1.0, 2.75])
+@pytest.mark.parametrize("mode", [0, 1])
+def test_codebook_matches_oracle(logq, bits, base, rng_, mode):
+    cb = logq.logq_build_codebook(bits, base, rng_, mode)
+    ocb = oracle.build_codebook(bits, base, rng_, mode)
+    qmax = ocb.qmax
+    half = 1 << (bits - 1)
+    assert cb.bits == bits and cb.qmax == qmax and cb.flags == mode
+    assert cb.base == base and cb.range == rng_
+    assert math.isclose(cb.shift, ocb.shift, rel_tol=0, abs_tol=1e-12)
+    lv = np.array(cb.level[: 2 * half], dtype=np.float32)
+    np.testing.assert_array_equal(lv[:half], ocb.levels32)
+    np.testing.assert_array_equal(lv[half:], -ocb.levels32)
+    assert np.signbit(lv[half])                          # code 1 << (n-1) is -0.0
+    np.testing.assert_array_equal(np.array(cb.thresh[:qmax], dtype=np.float32), ocb.taus32_up)
+    assert all(math.isinf(t) for t in cb.thresh[qmax:])
+    bf = np.array(cb.level_bf16[: 2 * half], dtype=np.uint16)
+    f16 = np.array(cb.level_f16[: 2 * half], dtype=np.uint16)
+    np.testing.assert_array_equal(bf[:half], ocb.levels_bf16_bits)
+    np.testing.assert_array_equal(bf[half:], ocb.levels_bf16_bits | 0x8000)
+    np.testing.assert_array_equal(f16[:half], ocb.levels_f16_bits)
+    np.testing.assert_array_equal(f16[half:], ocb.levels_f16_bits | 0x8000)
+
+
+@pytest.mark.parametrize("args", [(2, 1.5, 1.0, 0), (5, 1.5, 1.0, 0), (4, 1.0, 1.0, 0), (4, -2.0, 1.0, 0),
+                                  (4, float("inf"), 1.0, 0), (4, 1.5, 0.0, 0), (4, 1.5, -3.0, 0),
+                                  (4, 1.5, float("nan"), 0), (4, 1.5, 1.0, 2)])
+def test_codebook_invalid(logq, args):
+    with pytest.raises(logq.LogqError) as ei:
+        logq.logq_build_codebook(*args)
+    assert ei.value.status == logq.LOGQ_ERR_INVALID_ARG
+
+
+def test_codebook_null_out(logq):
+    assert logq.lib.logq_build_codebook(4, 1.5, 1.0, 0, None) == logq.LOGQ_ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("N,K,bits,want", [(512, 2048, 4, 512 * 1024), (3, 128, 3, 3 * 48),
+                                           (1, 128, 4, 64), (0, 128, 4, 0), (4, 100, 4, 0),
+                                           (4, 0, 4, 0), (4, 128, 5, 0), (-1, 128, 4, 0),
+                                           (14336, 4096, 3, 14336 * 1536)])
+def test_packed_bytes(logq, N, K, bits, want):
+    assert logq.logq_packed_bytes(N, K, bits) == want
+    if want:
+        assert want == N * oracle.packed_row_bytes(K, bits)
+
+
+def test_workspace_bytes(logq):
+    assert logq.logq_workspace_bytes() == 256
+
+
+def test_status_strings(logq):
+    for s in range(7):
+        assert len(logq.status_string(s)) >= 2
+    assert logq.status_string(99) == "unknown status"
+
+
+def _fake(addr):
+    return ctypes.c_void_p(addr)
+
+
+def test_quantize_rejects_before_launch(logq):
+    """Invalid requests fail in host validation (these run without a GPU:
+    nothing is enqueued, so the fake device addresses are never touched)."""
+    L = logq.lib
+    W, C, ws = _fake(0x10000), _fake(0x20000), _fake(0x30000)
+    cb = logq.Codebook()
+    ok_args = dict(N=4, K=128, bits=4, base=1.5, rng=1.0, flags=0)
+
+    def call(W=W, C=C, ws=ws, wsb=256, **kw):
+        a = dict(ok_args, **kw)
+        return L.logq_quantize(W, a["N"], a["K"], a["bits"], a["base"], a["rng"], a["flags"], C,
+                               ctypes.byref(cb), ws, wsb, None)
+
+    assert call(W=None) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(C=None) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(W=_fake(0x10004)) == logq.LOGQ_ERR_INVALID_ARG          # misaligned
+    assert call(K=100) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(N=0) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(bits=5) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(base=1.0) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(base=float("nan")) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(rng=float("inf")) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(flags=7) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(ws=None) == logq.LOGQ_ERR_WORKSPACE
+    assert call(wsb=16) == logq.LOGQ_ERR_WORKSPACE
+    assert call(ws=_fake(0x30008)) == logq.LOGQ_ERR_WORKSPACE
+
+
+def test_linear_rejects_before_launch(logq):
+    L = logq.lib
+    cb = logq.logq_build_codebook(4, 1.5, 1.0)
+    C, X, Y, ws = _fake(0x10000), _fake(0x20000), _fake(0x30000), _fake(0x40000)
+
+    def call(C=C, cbp=ctypes.byref(cb), X=X, xd=logq.LOGQ_BF16, B=1, N=8, K=128, Y=Y,
+             yd=logq.LOGQ_F32, ws=ws, wsb=256):
+        return L.logq_linear(C, cbp, X, xd, B, N, K, Y, yd, ws, wsb, None)
+
+    assert call(C=None) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(cbp=None) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(X=None) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(Y=_fake(0x30002)) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(B=0) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(K=96) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(N=-2) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(xd=logq.LOGQ_F32) == logq.LOGQ_ERR_UNSUPPORTED
+    assert call(xd=logq.LOGQ_BF16, yd=logq.LOGQ_F16) == logq.LOGQ_ERR_UNSUPPORTED
+    assert call(ws=None) == logq.LOGQ_ERR_WORKSPACE
+    assert call(wsb=255) == logq.LOGQ_ERR_WORKSPACE
+    bad = logq.logq_build_codebook(4, 1.5, 1.0)
+    bad.qmax = 3                                                     # inconsistent codebook
+    assert call(cbp=ctypes.byref(bad)) == logq.LOGQ_ERR_INVALID_ARG
+
+
+def test_workspace_status_rejects_null(logq):
+    assert logq.lib.logq_workspace_status(None, None, None) == logq.LOGQ_ERR_WORKSPACE

@@ -1,0 +1,161 @@
+"""Decode GEMV / skinny GEMM and prefill GEMM against the fp64 oracle:
+|y_gpu - y_ref| <= 1e-3 * sum_k |x_k w_k| + 1e-6 for every output, with the
+oracle evaluating X * What^T on the same codes and the same 16-bit table."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2607_01127_gb300 import workloads
+
+from gpu_common import check_linear, lib
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def logq():
+    return lib()
+
+
+def make_layer(logq, N, K, bits, base, seed, outliers=False):
+    w = workloads.weights_np(N, K, seed, outliers=outliers)
+    codes, cb = logq.logq_quantize(torch.from_numpy(w).cuda(), bits, base)
+    ocb = oracle.build_codebook(bits, base, cb.range)
+    q = oracle.unpack(codes.cpu().numpy().reshape(N, -1), N, K, bits)
+    return codes, cb, ocb, q
+
+
+def reference(X, q, ocb):
+    table = oracle.TABLE_BF16 if X.dtype == torch.bfloat16 else oracle.TABLE_F16
+    return oracle.linear(X.float().cpu().double().numpy(), oracle.dequant(q, ocb, table), nthreads=0)
+
+
+def run_case(logq, N, K, bits, B, xdt, ydt=None, seed=0, base=1.5):
+    codes, cb, ocb, q = make_layer(logq, N, K, bits, base, seed)
+    X = workloads.activations_torch(B, K, seed, xdt, "cuda")
+    Y = logq.logq_linear(codes, cb, X, N, K, y_dtype=ydt)
+    Yr, A = reference(X, q, ocb)
+    name = {None: "f32", torch.float32: "f32", torch.bfloat16: "bf16", torch.float16: "f16"}[ydt]
+    return check_linear(Y.double().cpu().numpy(), Yr, A, name)
+
+
+@pytest.mark.parametrize("N,K", [(512, 2048), (7, 128), (300, 1152), (1000, 4096), (129, 14336),
+                                 (2049, 384)])
+@pytest.mark.parametrize("B", [1, 2, 3, 4, 5, 8, 16])
+def test_gemv_4bit_bf16(logq, N, K, B):
+    run_case(logq, N, K, 4, B, torch.bfloat16, seed=N + K + B)
+
+
+@pytest.mark.parametrize("N,K", [(512, 2048), (7, 128), (300, 1152), (129, 14336)])
+@pytest.mark.parametrize("B", [1, 2, 3, 4])
+def test_gemv_3bit_bf16(logq, N, K, B):
+    run_case(logq, N, K, 3, B, torch.bfloat16, seed=N + K + B, base=1.25)
+
+
+@pytest.mark.parametrize("bits,B", [(4, 1), (4, 4), (4, 16), (3, 1), (3, 4)])
+def test_gemv_fp16_activations(logq, bits, B):
+    run_case(logq, 512, 2048, bits, B, torch.float16, seed=B)
+
+
+@pytest.mark.parametrize("xdt", [torch.bfloat16, torch.float16])
+@pytest.mark.parametrize("B", [1, 4, 16])
+def test_gemv_16bit_output(logq, xdt, B):
+    run_case(logq, 384, 1024, 4, B, xdt, ydt=xdt, seed=3)
+
+
+def test_gemv_config_single_layer(logq):
+    """512 x 2048 layer, fp16 x [1, 2048], b = 1.5, seed 0."""
+    run_case(logq, 512, 2048, 4, 1, torch.float16, seed=0)
+
+
+@pytest.mark.parametrize("bits", [3, 4])
+def test_one_hot_returns_decoded_column(logq, bits):
+    """x = e_k picks column k of What exactly (pins the code layout)."""
+    N, K = 96, 256
+    codes, cb, ocb, q = make_layer(logq, N, K, bits, 1.5, 4)
+    wq = oracle.dequant(q, ocb, oracle.TABLE_BF16)
+    for k in (0, 1, 2, 31, 32, 33, 127, 200, 255):
+        X = torch.zeros(1, K, dtype=torch.bfloat16, device="cuda")
+        X[0, k] = 1.0
+        Y = logq.logq_linear(codes, cb, X, N, K).double().cpu().numpy()[0]
+        np.testing.assert_array_equal(Y, wq[:, k])
+
+
+def test_zero_and_ones(logq):
+    N, K = 64, 512
+    codes, cb, ocb, q = make_layer(logq, N, K, 4, 1.5, 8)
+    Y0 = logq.logq_linear(codes, cb, torch.zeros(3, K, dtype=torch.bfloat16, device="cuda"), N, K)
+    assert torch.count_nonzero(Y0) == 0
+    X1 = torch.ones(1, K, dtype=torch.bfloat16, device="cuda")
+    Y1 = logq.logq_linear(codes, cb, X1, N, K).double().cpu().numpy()[0]
+    rows = oracle.dequant(q, ocb, oracle.TABLE_BF16)
+    check_linear(Y1[None], rows.sum(1)[None], np.abs(rows).sum(1)[None])
+
+
+def test_hand_written_codes(logq):
+    """Codes written by hand (not by the quantiser): row n holds code c(n) at
+    every k, so y[n] = table[c(n)] * sum_k x_k."""
+    K = 256
+    cb = logq.logq_build_codebook(4, 2.0, 1.0)     # levels 2^(m-7), exact in bf16
+    codes = np.zeros((16, K // 2), np.uint8)
+    for c in range(16):
+        codes[c, :] = c | (c << 4)
+    X = torch.full((1, K), 0.5, dtype=torch.bfloat16, device="cuda")
+    Y = logq.logq_linear(torch.from_numpy(codes.reshape(-1)).cuda(), cb, X, 16, K).cpu().numpy()[0]
+    want = np.array([cb.level[c] * 0.5 * K for c in range(16)], dtype=np.float32)
+    np.testing.assert_array_equal(Y, want)
+
+
+def test_gemv_repeatable_and_stream(logq):
+    N, K = 4096, 4096
+    codes, cb, ocb, q = make_layer(logq, N, K, 4, 1.5, 1)
+    X = workloads.activations_torch(1, K, 1, torch.bfloat16, "cuda")
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        Ya = logq.logq_linear(codes, cb, X, N, K)
+        Yb = logq.logq_linear(codes, cb, X, N, K)
+    s.synchronize()
+    assert torch.equal(Ya, Yb)                        # deterministic reduction order
+
+
+def test_gemv_cuda_graph_capture(logq):
+    N, K = 2048, 2048
+    codes, cb, ocb, q = make_layer(logq, N, K, 4, 1.5, 2)
+    X = workloads.activations_torch(1, K, 2, torch.bfloat16, "cuda")
+    Y = torch.empty(1, N, device="cuda")
+    ws = logq.new_workspace()
+    logq.logq_linear(codes, cb, X, N, K, Y=Y, workspace=ws)          # warm-up outside capture
+    g = torch.cuda.CUDAGraph()
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        with torch.cuda.graph(g, stream=s):
+            logq.logq_linear(codes, cb, X, N, K, Y=Y, workspace=ws)
+    Y.zero_()
+    g.replay()
+    torch.cuda.synchronize()
+    Yr, A = reference(X, q, ocb)
+    check_linear(Y.double().cpu().numpy(), Yr, A)
+
+
+@pytest.mark.parametrize("N,K,B", [(256, 512, 128), (300, 1152, 200), (1024, 2048, 256), (512, 4096, 2048),
+                                   (4096, 4096, 256), (200, 128, 17)])
+@pytest.mark.parametrize("bits", [3, 4])
+def test_prefill_bf16(logq, N, K, B, bits):
+    run_case(logq, N, K, bits, B, torch.bfloat16, seed=N + B + bits)
+
+
+@pytest.mark.parametrize("ydt", [torch.bfloat16, None])
+def test_prefill_output_dtypes_and_fp16(logq, ydt):
+    run_case(logq, 512, 1024, 4, 256, torch.bfloat16, ydt=ydt, seed=5)
+    run_case(logq, 512, 1024, 4, 256, torch.float16, ydt=None, seed=6)
+
+
+def test_prefill_workspace_status_clean(logq):
+    N, K, B = 1024, 2048, 512
+    codes, cb, ocb, q = make_layer(logq, N, K, 4, 1.5, 9)
+    ws = logq.new_workspace()
+    X = workloads.activations_torch(B, K, 9, torch.bfloat16, "cuda")
+    logq.logq_linear(codes, cb, X, N, K, workspace=ws)
+    st, detail = logq.logq_workspace_status(ws)
+    assert st == logq.LOGQ_OK and detail == 0
