@@ -154,6 +154,28 @@ logq_status logq_linear(const uint8_t* codes, const logq_codebook* cb, const voi
                         logq_dtype y_dtype, void* workspace, size_t workspace_bytes,
                         void* stream);
 
+/*
+ * Allocation-free variant of logq_quantize (the paper has no counterpart; it
+ * serves callers of this library that must not allocate device memory, such as
+ * a plugin whose host application owns all device memory through its own pool,
+ * or a latency-critical path that cannot take the device synchronisation an
+ * allocation implies -- and that therefore cannot supply a workspace).
+ * Instead of a caller workspace it uses a 256-byte scratch record kept in a
+ * static device array of the library; each GPU that loads the library holds
+ * that array until the process exits.  The scratch does not grow with N or K,
+ * so the call accepts every size logq_quantize accepts (LOGQ_ERR_WORKSPACE would
+ * report a scratch need beyond the array).  It calls no cudaMalloc, cudaFree
+ * or other allocating routine.  Its first call on a device looks up the array's
+ * device address (with that device current); make that first call before any
+ * stream capture.  All calls share the one array, which keeps the last call's
+ * contents (each call clears the words it needs): calls that overlap on the
+ * GPU race and must be serialised by the caller.  Arguments, the single stream
+ * synchronisation and the errors are otherwise those of logq_quantize.
+ */
+logq_status logq_quantize_noalloc(const float* W, int64_t N, int64_t K, int bits, double base,
+                                  double range, int flags, uint8_t* codes,
+                                  logq_codebook* cb_out, void* stream);
+
 /* Synchronise `stream`, read the device error word of `workspace`, clear it,
  * and return LOGQ_OK or LOGQ_ERR_TIMEOUT.  *detail (host, may be NULL)
  * receives an implementation code naming the wait that gave up. */

@@ -37,7 +37,8 @@ LOGQ_F32, LOGQ_BF16, LOGQ_F16 = 0, 1, 2
 LOGQ_SHIFT_EXACT, LOGQ_SHIFT_FLOOR = 0, 1
 
 EXPORTED = ("logq_build_codebook", "logq_packed_bytes", "logq_workspace_bytes", "logq_quantize",
-            "logq_linear", "logq_workspace_status", "logq_status_string", "logq_device_sm_count")
+            "logq_linear", "logq_workspace_status", "logq_status_string", "logq_device_sm_count",
+            "logq_quantize_noalloc")
 
 
 class Codebook(ctypes.Structure):
@@ -77,6 +78,9 @@ def _load() -> ctypes.CDLL:
     lib.logq_quantize.argtypes = [P, c_i64, c_i64, c_int, c_dbl, c_dbl, c_int, P,
                                   ctypes.POINTER(Codebook), P, ctypes.c_size_t, P]
     lib.logq_quantize.restype = c_int
+    lib.logq_quantize_noalloc.argtypes = [P, c_i64, c_i64, c_int, c_dbl, c_dbl, c_int, P,
+                                          ctypes.POINTER(Codebook), P]
+    lib.logq_quantize_noalloc.restype = c_int
     lib.logq_linear.argtypes = [P, ctypes.POINTER(Codebook), P, c_int, c_i64, c_i64, c_i64, P,
                                 c_int, P, ctypes.c_size_t, P]
     lib.logq_linear.restype = c_int
@@ -171,6 +175,23 @@ def logq_quantize(W, bits: int, base: float, range_: float = 0.0, flags: int = L
                            int(flags), ctypes.c_void_p(codes.data_ptr()), ctypes.byref(cb),
                            ctypes.c_void_p(workspace.data_ptr()), workspace.numel(), _stream_ptr(stream))
     _check(st, "logq_quantize")
+    return codes[:nbytes], cb
+
+
+def logq_quantize_noalloc(W, bits: int, base: float, range_: float = 0.0,
+                          flags: int = LOGQ_SHIFT_EXACT, codes=None, stream=None):
+    """logq_quantize without a caller workspace (static device scratch; see logq.h)."""
+    import torch
+    assert W.dtype == torch.float32 and W.is_cuda and W.dim() == 2 and W.is_contiguous()
+    N, K = W.shape
+    nbytes = logq_packed_bytes(N, K, bits)
+    if codes is None:
+        codes = torch.empty(max(nbytes, 16), dtype=torch.uint8, device=W.device)
+    cb = Codebook()
+    st = _lib().logq_quantize_noalloc(ctypes.c_void_p(W.data_ptr()), N, K, int(bits), float(base),
+                                      float(range_), int(flags), ctypes.c_void_p(codes.data_ptr()),
+                                      ctypes.byref(cb), _stream_ptr(stream))
+    _check(st, "logq_quantize_noalloc")
     return codes[:nbytes], cb
 
 
