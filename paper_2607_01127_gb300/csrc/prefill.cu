@@ -1,6 +1,636 @@
-// Prefill GEMM (tcgen05) -- placeholder until the tensor-core kernel lands.
+// Prefill GEMM on the tensor cores: Y[t][n] = sum_k X[t][k] * table[code(n, k)]
+// (paper Sec. 3.3; the paper attributes its large-batch slowdown to per-element
+// LUT reads, so here each weight is dequantised once per tile and reused by a
+// dense bf16/fp16 contraction).
+//
+// One persistent CTA per SM walks 128 (weights) x 256 (tokens) output tiles.
+// Warp roles:
+//   warp 0     TMA producer: X tiles [256 tokens x 64 k] with 128-byte swizzle.
+//   warp 1     MMA issuer: tcgen05.mma kind::f16, M = 128 (weight rows),
+//              N = 256 (tokens), K = 16, fp32 accumulators in tensor memory,
+//              double-buffered (2 x 256 columns), so the epilogue of one tile
+//              overlaps the main loop of the next.  Also allocates TMEM.
+//   warps 2-5  epilogue: tcgen05.ld of the accumulator, stores of Y (each warp
+//              reads its TMEM lane quarter; lane n writes Y[t][n0 + n]).
+//   warps 6-13 decode: two threads per weight row of the tile, each owning 32
+//              of the stage's 64 k; a thread streams its codes into its own
+//              16-byte slot of a shared ring with cp.async, resolves two codes
+//              per lookup in a per-lane-replicated pair table, and writes the
+//              bf16 (or fp16) weight tile into shared memory in the K-major
+//              128-byte-swizzled layout the MMA reads, followed by a proxy fence.
+// Every mbarrier wait is bounded: a wait that exceeds ~1 s of clock cycles
+// raises an abort flag, records LOGQ_ERR_TIMEOUT in the caller's workspace and
+// lets every role leave its loop; the kernel drains what it issued, frees its
+// tensor memory and returns.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cudaTypedefs.h>
+#include <stdint.h>
+#include <string.h>
+
+#include <mutex>
+
 #include "internal.h"
 
 namespace logq {
-cudaError_t launch_prefill(const LinearArgs&, cudaStream_t) { return cudaErrorNotSupported; }
+namespace {
+
+constexpr int kBM = 128;                 // weight rows per tile (MMA M)
+constexpr int kBN = 256;                 // tokens per tile (MMA N)
+constexpr int kBK = 64;                  // k per stage (one 128-byte swizzle atom of bf16)
+constexpr int kStages = 3;
+constexpr int kCodeRing = 7;             // code stages in flight per decode thread
+constexpr int kDecodeWarps = 8;
+constexpr int kDecodeThreads = 32 * kDecodeWarps;  // two threads per weight row
+constexpr int kThreads = 32 * (6 + kDecodeWarps);  // producer, MMA, 4 epilogue, decode
+constexpr int kXStageBytes = kBN * kBK * 2;      // 32 KiB
+constexpr int kWStageBytes = kBM * kBK * 2;      // 16 KiB
+constexpr int kCodeSlotBytes = 16;               // codes of half a row and stage (<= 16 B)
+constexpr int kCodeStageBytes = kDecodeThreads * kCodeSlotBytes;
+constexpr int kTabBytes4 = 256 * 128;            // 4-bit pair table, 32 copies
+constexpr uint32_t kTmemCols = 2 * kBN;          // two fp32 accumulators
+constexpr long long kWaitLimit = 2000000000LL;   // cycles (~1 s)
+
+// error detail codes (workspace->detail)
+enum : uint32_t { kWaitProducer = 1, kWaitMma = 2, kWaitEpilogue = 3, kWaitDecode = 4, kWaitDrain = 5,
+                  kWaitLayout = 6 };
+
+struct PrefillParams {
+    const uint8_t* codes;
+    void* Y;
+    Workspace* ws;
+    int64_t N;
+    int32_t K, B;
+    int64_t row_bytes;
+    int32_t bits;
+    int32_t y_dtype;
+    int32_t n_tiles_n, n_tiles_t;
+    uint32_t idesc;
+    uint32_t smem_bytes;    // dynamic shared memory of the launch (layout check)
+    uint32_t lvl16[16];
+};
+
+// ------------------------------------------------------------------ PTX ---
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count)
+{
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar)
+{
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes)
+{
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Bounded wait, slow path: polls until the phase completes, the abort flag
+// rises (unless draining) or ~1 s of cycles pass; running out raises the
+// abort flag and records LOGQ_ERR_TIMEOUT in the workspace.
+__device__ __noinline__ bool wait_slow(uint32_t bar, uint32_t parity, volatile int* abort_flag, Workspace* ws,
+                                       uint32_t who, bool drain)
+{
+    const long long t0 = clock64();
+    for (;;) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if (!drain && *abort_flag) return false;
+        if (clock64() - t0 > kWaitLimit) {
+            *abort_flag = 1;
+            atomicExch(&ws->detail, who);
+            atomicExch(&ws->error, (uint32_t)LOGQ_ERR_TIMEOUT);
+            return false;
+        }
+    }
+}
+
+__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                             Workspace* ws, uint32_t who, bool drain = false)
+{
+    if (mbar_try_wait(bar, parity)) return true;
+    return wait_slow(bar, parity, abort_flag, ws, who, drain);
+}
+
+// One lane of the warp polls (a barrier polled by many threads serialises);
+// the outcome is broadcast to the whole warp.
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag, Workspace* ws,
+                                          uint32_t who)
+{
+    uint32_t ok = 0;
+    if ((threadIdx.x & 31) == 0) ok = wait_bounded(bar, parity, abort_flag, ws, who) ? 1u : 0u;
+    return __shfl_sync(0xffffffffu, ok, 0) != 0;
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
+        ::"r"(dst), "l"(map), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void cp_async_4(uint32_t dst, const void* src)
+{
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(dst), "l"(src) : "memory");
+}
+
+__device__ __forceinline__ void cp_async_8(uint32_t dst, const void* src)
+{
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(dst), "l"(src) : "memory");
+}
+
+__device__ __forceinline__ void cp_async_16(uint32_t dst, const void* src)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, rows of
+// 128 bytes, 8-row groups 1024 bytes apart (stride byte offset), version 1.
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t addr)
+{
+    uint64_t d = 0;
+    d |= (uint64_t)((addr & 0x3ffffu) >> 4);          // start address
+    d |= (uint64_t)1 << 16;                            // leading byte offset (unused for this layout)
+    d |= (uint64_t)(1024 >> 4) << 32;                  // stride byte offset
+    d |= (uint64_t)1 << 46;                            // descriptor version
+    d |= (uint64_t)2 << 61;                            // swizzle: 128 bytes
+    return d;
+}
+
+__device__ __forceinline__ void mma_f16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                        uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+        ::"r"(tmem_d), "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint32_t bar)
+{
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+                 : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32])
+{
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr)
+        : "memory");
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t lds32(uint32_t addr)
+{
+    uint32_t v;
+    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr));
+    return v;
+}
+
+__device__ __forceinline__ uint4 lds128(uint32_t addr)
+{
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
+    return v;
+}
+
+__device__ __forceinline__ void sts128(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d)
+{
+    asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d)
+                 : "memory");
+}
+
+__device__ __forceinline__ void store_y(void* Y, int dtype, int64_t idx, float v)
+{
+    if (dtype == LOGQ_F32) static_cast<float*>(Y)[idx] = v;
+    else if (dtype == LOGQ_BF16) static_cast<__nv_bfloat16*>(Y)[idx] = __float2bfloat16_rn(v);
+    else static_cast<__half*>(Y)[idx] = __float2half_rn(v);
+}
+
+// ------------------------------------------------------------------ kernel ---
+
+__global__ void __launch_bounds__(kThreads, 1)
+prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ CUtensorMap xmap)
+{
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    // Layout: the pair table sits at the first 32 KiB-aligned shared address
+    // (so a lookup address is an OR of fields); the code ring and barriers use
+    // the space below it when it is large enough, else they follow the stages.
+    //   [code ring | barriers | pad] table (32 KiB) | X stages | W stages [| code ring | barriers]
+    const uint32_t sbase = smem_u32(smem_raw);
+    const uint32_t tab = (sbase + 32767u) & ~32767u;
+    const uint32_t xs0 = tab + kTabBytes4;
+    const uint32_t ws0 = xs0 + kStages * kXStageBytes;
+    constexpr uint32_t kLowBytes = kCodeRing * kCodeStageBytes + 256;
+    const bool low = tab - sbase >= kLowBytes;
+    const uint32_t cr0 = low ? sbase : ws0 + kStages * kWStageBytes;
+    const uint32_t bar0 = cr0 + kCodeRing * kCodeStageBytes;
+    const uint32_t layout_end = low ? ws0 + kStages * kWStageBytes : bar0 + 256;
+    if (layout_end > sbase + p.smem_bytes) {          // launch too small for this layout: refuse
+        if (threadIdx.x == 0) {
+            atomicExch(&p.ws->detail, (uint32_t)kWaitLayout);
+            atomicExch(&p.ws->error, (uint32_t)LOGQ_ERR_TIMEOUT);
+        }
+        return;
+    }
+    uint8_t* gen = smem_raw - sbase;                  // generic pointer = gen + shared address
+    // barriers: xfull[S], wfull[S], empty[S], accfull[2], accempty[2], then tmem slot and abort flag
+    auto xfull = [&](int s) { return bar0 + 8u * s; };
+    auto wfull = [&](int s) { return bar0 + 8u * (kStages + s); };
+    auto empty = [&](int s) { return bar0 + 8u * (2 * kStages + s); };
+    auto accfull = [&](int b) { return bar0 + 8u * (3 * kStages + b); };
+    auto accempty = [&](int b) { return bar0 + 8u * (3 * kStages + 2 + b); };
+    const uint32_t drainb = bar0 + 8u * (3 * kStages + 4);
+    const uint32_t tmem_slot = bar0 + 8u * (3 * kStages + 5);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(gen + tmem_slot + 8);
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    if (tid == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(xfull(s), 1);
+            mbar_init(wfull(s), kDecodeWarps);
+            mbar_init(empty(s), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(accfull(b), 1);
+            mbar_init(accempty(b), 4);
+        }
+        mbar_init(drainb, 1);
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(&xmap) : "memory");
+    }
+    // pair table: entry e (two codes) = bf16x2 / f16x2 of their levels, one copy per lane
+    {
+        const int nent = (p.bits == 4) ? 256 : 64;
+        for (int i = tid; i < nent * 8; i += kThreads) {
+            const int e = i >> 3, part = i & 7;
+            const uint32_t lo = (p.bits == 4) ? (e & 15) : (e & 7);
+            const uint32_t hi = (p.bits == 4) ? (e >> 4) : (e >> 3);
+            const uint32_t v = (p.lvl16[lo] & 0xffffu) | (p.lvl16[hi] << 16);
+            sts128(tab + e * 128 + part * 16, v, v, v, v);
+        }
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(tmem_slot),
+                     "r"(kTmemCols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *reinterpret_cast<volatile uint32_t*>(gen + tmem_slot);
+
+    const int ksteps = p.K / kBK;
+    const int ntiles = p.n_tiles_n * p.n_tiles_t;
+
+    if (warp == 0) {
+        // ---------------- TMA producer ----------------
+        if (lane == 0) {
+            int stage = 0;
+            uint32_t phase = 0;
+            bool ok = true;
+            uint32_t issued = 0, issued_par = 0;       // per stage: used at least once / parity of last load
+            // the code rows of a tile are one contiguous block: ask L2 for it one
+            // tile ahead so the decode warps' copies hit L2
+            auto prefetch_codes = [&](int tile) {
+                if (tile >= ntiles) return;
+                const int64_t n0 = (int64_t)(tile % p.n_tiles_n) * kBM;
+                const int64_t rows = (p.N - n0) < kBM ? (p.N - n0) : kBM;
+                const uint8_t* base = p.codes + n0 * p.row_bytes;
+                const int64_t bytes = rows * p.row_bytes;
+                for (int64_t off = 0; off < bytes; off += 16384) {
+                    const int64_t nb = (bytes - off) < 16384 ? (bytes - off) : 16384;
+                    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base + off), "r"((uint32_t)nb)
+                                 : "memory");
+                }
+            };
+            prefetch_codes(blockIdx.x);
+            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+                const int t0 = (tile / p.n_tiles_n) * kBN;
+                prefetch_codes(tile + gridDim.x);
+                for (int ks = 0; ks < ksteps; ++ks) {
+                    if (!wait_bounded(empty(stage), phase ^ 1u, abort_flag, p.ws, kWaitProducer)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_expect_tx(xfull(stage), kXStageBytes);
+                    tma_load_2d(xs0 + stage * kXStageBytes, &xmap, ks * kBK, t0, xfull(stage));
+                    issued |= 1u << stage;
+                    issued_par = (issued_par & ~(1u << stage)) | (phase << stage);
+                    if (++stage == kStages) { stage = 0; phase ^= 1u; }
+                }
+            }
+            // every load this thread issued has landed before the CTA can leave
+            for (int st = 0; st < kStages; ++st)
+                if (issued & (1u << st))
+                    wait_bounded(xfull(st), (issued_par >> st) & 1u, abort_flag, p.ws, kWaitDrain, true);
+        }
+    } else if (warp == 1) {
+        // ---------------- MMA issuer ----------------
+        if (lane == 0) {
+            int stage = 0;
+            uint32_t phase = 0;
+            bool ok = true;
+            int it = 0;
+            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
+                const int buf = it & 1;
+                const uint32_t acc_phase = ((uint32_t)it >> 1) & 1u;
+                if (!wait_bounded(accempty(buf), acc_phase ^ 1u, abort_flag, p.ws, kWaitMma)) break;
+                tc_fence_after();
+                const uint32_t dcol = tmem_base + (uint32_t)(buf * kBN);
+                for (int ks = 0; ks < ksteps; ++ks) {
+                    if (!wait_bounded(xfull(stage), phase, abort_flag, p.ws, kWaitMma) ||
+                        !wait_bounded(wfull(stage), phase, abort_flag, p.ws, kWaitMma)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint64_t adesc = smem_desc_sw128(ws0 + stage * kWStageBytes);
+                    const uint64_t bdesc = smem_desc_sw128(xs0 + stage * kXStageBytes);
+#pragma unroll
+                    for (int kk = 0; kk < kBK / 16; ++kk) {
+                        // 16 k of bf16 = 32 bytes (2 descriptor units) further inside the swizzle atom
+                        mma_f16(dcol, adesc + 2 * kk, bdesc + 2 * kk, p.idesc, (ks | kk) != 0);
+                    }
+                    mma_commit(empty(stage));
+                    if (++stage == kStages) { stage = 0; phase ^= 1u; }
+                }
+                if (ok) mma_commit(accfull(buf));
+            }
+        }
+    } else if (warp >= 2 && warp < 6) {
+        // ---------------- epilogue ----------------
+        const int quarter = warp & 3;                   // TMEM lanes 32*quarter .. +31
+        const int row = quarter * 32 + lane;
+        int it = 0;
+        for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
+            const int buf = it & 1;
+            const uint32_t acc_phase = ((uint32_t)it >> 1) & 1u;
+            if (!warp_wait(accfull(buf), acc_phase, abort_flag, p.ws, kWaitEpilogue)) break;
+            tc_fence_after();
+            const int64_t n = (int64_t)(tile % p.n_tiles_n) * kBM + row;
+            const int t0 = (tile / p.n_tiles_n) * kBN;
+#pragma unroll 1
+            for (int c = 0; c < kBN / 32; ++c) {
+                uint32_t v[32];
+                tmem_ld32(tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * kBN + c * 32), v);
+                if (n < p.N) {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        const int t = t0 + c * 32 + j;
+                        if (t < p.B) store_y(p.Y, p.y_dtype, (int64_t)t * p.N + n, __uint_as_float(v[j]));
+                    }
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(accempty(buf));
+        }
+    } else {
+        // ---------------- decode ----------------
+        const int d = tid - 6 * 32;                     // 0 .. kDecodeThreads-1
+        const int r = d & (kBM - 1);                    // weight row within the tile
+        const int h = d >> 7;                           // half: k 32h .. 32h+31 of the stage
+        const uint32_t tl = tab | (4u * (uint32_t)lane);
+        const int hbytes = (p.bits == 4) ? 16 : 12;     // codes of one half row per stage
+        int stage = 0;
+        uint32_t phase = 0;
+        const int my_tiles = (ntiles > (int)blockIdx.x) ? (ntiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
+        const int total = my_tiles * ksteps;            // stages this CTA decodes
+        // Cursor over (tile, k-step) advanced without divisions: one for the
+        // copies issued ahead, one for the stage being decoded.
+        struct Cursor {
+            int tile, ks;
+            bool valid;                                 // this thread's row exists
+            const uint8_t* row;                         // its codes, half h, stage 0
+        };
+        auto set_tile = [&](Cursor& c, int tile) {
+            c.tile = tile;
+            c.ks = 0;
+            const int64_t n = (int64_t)(tile % p.n_tiles_n) * kBM + r;
+            c.valid = tile < ntiles && n < p.N;
+            c.row = p.codes + (c.valid ? n : 0) * p.row_bytes + (int64_t)h * hbytes;
+        };
+        auto step = [&](Cursor& c) {
+            if (++c.ks == ksteps) set_tile(c, c.tile + (int)gridDim.x);
+        };
+        Cursor ahead, cur;
+        set_tile(ahead, (int)blockIdx.x);
+        set_tile(cur, (int)blockIdx.x);
+        auto issue = [&](int g) {
+            if (g < total && ahead.valid) {
+                const uint8_t* src = ahead.row + (int64_t)ahead.ks * (2 * hbytes);
+                const uint32_t dst = cr0 + (g % kCodeRing) * kCodeStageBytes + d * kCodeSlotBytes;
+                if (p.bits == 4) {
+                    cp_async_16(dst, src);
+                } else {
+                    cp_async_4(dst, src);
+                    cp_async_4(dst + 4, src + 4);
+                    cp_async_4(dst + 8, src + 8);
+                }
+            }
+            if (g < total) step(ahead);
+            cp_async_commit();
+        };
+        for (int g = 0; g < kCodeRing - 1; ++g) issue(g);
+        int slot = 0;                                   // g % kCodeRing
+        for (int g = 0; g < total; ++g) {
+            issue(g + kCodeRing - 1);
+            cp_async_wait<kCodeRing - 1>();
+            const bool valid = cur.valid;
+            uint4 cv = make_uint4(0, 0, 0, 0);
+            if (valid) cv = lds128(cr0 + slot * kCodeStageBytes + d * kCodeSlotBytes);
+            if (++slot == kCodeRing) slot = 0;
+            step(cur);
+            const uint32_t cw[4] = {cv.x, cv.y, cv.z, cv.w};
+            if (!warp_wait(empty(stage), phase ^ 1u, abort_flag, p.ws, kWaitDecode)) break;
+            const uint32_t wrow = ws0 + stage * kWStageBytes + r * 128;
+            const uint32_t sw = (uint32_t)(r & 7);
+            if (p.bits == 4) {
+                // word i holds k = 32h + 8i .. +7 -> 16-byte chunk 4h + i of the row
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const uint32_t c = cw[i];
+                    const uint32_t a0 = lds32(((c << 7) & 0x7f80u) | tl);
+                    const uint32_t a1 = lds32(((c >> 1) & 0x7f80u) | tl);
+                    const uint32_t a2 = lds32(((c >> 9) & 0x7f80u) | tl);
+                    const uint32_t a3 = lds32(((c >> 17) & 0x7f80u) | tl);
+                    sts128(wrow + ((((uint32_t)(4 * h + i)) ^ sw) << 4), a0, a1, a2, a3);
+                }
+            } else {
+                // one 12-byte group of 32 k; pair p -> chunk 4h + p / 4
+                uint32_t pr[16];
+#pragma unroll
+                for (int i = 0; i < 3; ++i) {
+                    pr[5 * i + 0] = lds32(((cw[i] << 7) & 0x1f80u) | tl);
+                    pr[5 * i + 1] = lds32(((cw[i] << 1) & 0x1f80u) | tl);
+                    pr[5 * i + 2] = lds32(((cw[i] >> 5) & 0x1f80u) | tl);
+                    pr[5 * i + 3] = lds32(((cw[i] >> 11) & 0x1f80u) | tl);
+                    pr[5 * i + 4] = lds32(((cw[i] >> 17) & 0x1f80u) | tl);
+                }
+                pr[15] = lds32(((cw[0] >> 23) & 0x0180u) | ((cw[1] >> 21) & 0x0600u) | ((cw[2] >> 19) & 0x1800u) | tl);
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    sts128(wrow + ((((uint32_t)(4 * h + i)) ^ sw) << 4), pr[4 * i], pr[4 * i + 1], pr[4 * i + 2],
+                           pr[4 * i + 3]);
+            }
+            fence_proxy_async();          // this thread's tile writes -> visible to the tensor core
+            __syncwarp();
+            if (lane == 0) mbar_arrive(wfull(stage));
+            if (++stage == kStages) { stage = 0; phase ^= 1u; }
+        }
+        cp_async_wait<0>();
+    }
+
+    // teardown: every MMA this CTA issued has completed before TMEM is freed
+    __syncthreads();
+    if (warp == 1) {
+        if (lane == 0) {
+            mma_commit(drainb);
+            wait_bounded(drainb, 0, abort_flag, p.ws, kWaitDrain, true);
+        }
+        __syncwarp();
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(kTmemCols)
+                     : "memory");
+    }
+}
+
+// ------------------------------------------------------------------ host ---
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+    });
+    return fn;
+}
+
+uint32_t make_idesc(bool f16_inputs)
+{
+    uint32_t d = 0;
+    d |= 1u << 4;                                   // D format: fp32
+    const uint32_t ab = f16_inputs ? 0u : 1u;       // A/B format: fp16 = 0, bf16 = 1
+    d |= ab << 7;
+    d |= ab << 10;
+    // bits 15, 16: A and B K-major (0)
+    d |= (uint32_t)(kBN >> 3) << 17;                // N / 8
+    d |= (uint32_t)(kBM >> 4) << 24;                // M / 16
+    return d;
+}
+
+constexpr uint32_t kStageRegion = kStages * (kXStageBytes + kWStageBytes);
+constexpr uint32_t kRingRegion = kCodeRing * kCodeStageBytes + 256;
+
+// Dynamic shared memory for the layout above, given where the dynamic region
+// starts in the CTA's shared window (after the reserved shared memory).
+uint32_t smem_bytes_for(uint32_t start)
+{
+    const uint32_t pad = (32768u - (start & 32767u)) & 32767u;
+    return pad >= kRingRegion ? pad + kTabBytes4 + kStageRegion : pad + kTabBytes4 + kStageRegion + kRingRegion;
+}
+
+}  // namespace
+
+cudaError_t launch_prefill(const LinearArgs& a, cudaStream_t s)
+{
+    auto encode = encode_fn();
+    if (!encode) return cudaErrorNotSupported;
+    CUtensorMap xmap;
+    memset(&xmap, 0, sizeof xmap);
+    const cuuint64_t gdim[2] = {(cuuint64_t)a.K, (cuuint64_t)a.B};
+    const cuuint64_t gstride[1] = {(cuuint64_t)a.K * 2};
+    const cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)kBN};
+    const cuuint32_t estride[2] = {1, 1};
+    CUresult r = encode(&xmap, a.x_f16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                        const_cast<void*>(a.X), gdim, gstride, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+
+    PrefillParams p;
+    memset(&p, 0, sizeof p);
+    p.codes = a.codes;
+    p.Y = a.Y;
+    p.ws = a.ws;
+    p.N = a.N;
+    p.K = (int32_t)a.K;
+    p.B = (int32_t)a.B;
+    p.bits = a.bits;
+    p.row_bytes = (a.bits == 4) ? a.K / 2 : a.K / 32 * 12;
+    p.y_dtype = a.y_dtype;
+    p.n_tiles_n = (int32_t)((a.N + kBM - 1) / kBM);
+    p.n_tiles_t = (int32_t)((a.B + kBN - 1) / kBN);
+    p.idesc = make_idesc(a.x_f16 != 0);
+    for (int c = 0; c < 16; ++c) p.lvl16[c] = a.lvl16[c];
+    const int64_t ntiles = (int64_t)p.n_tiles_n * p.n_tiles_t;
+    const int sms = sm_count() > 0 ? sm_count() : 148;
+    const int grid = (int)(ntiles < sms ? ntiles : sms);
+
+    static uint32_t configured[64] = {0};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    if (!configured[dev]) {
+        int reserved = 0, optin = 0;
+        if ((e = cudaDeviceGetAttribute(&reserved, cudaDevAttrReservedSharedMemoryPerBlock, dev)) != cudaSuccess) return e;
+        if ((e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev)) != cudaSuccess) return e;
+        const uint32_t bytes = smem_bytes_for((uint32_t)reserved);
+        if (bytes > (uint32_t)optin) return cudaErrorNotSupported;
+        e = cudaFuncSetAttribute(prefill_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+        if (e != cudaSuccess) return e;
+        configured[dev] = bytes;
+    }
+    p.smem_bytes = configured[dev];
+    prefill_kernel<<<grid, kThreads, configured[dev], s>>>(p, xmap);
+    return cudaGetLastError();
+}
+
 }  // namespace logq
