@@ -39,7 +39,8 @@ namespace {
 constexpr int kBM = 128;                 // weight rows per tile (MMA M)
 constexpr int kBN = 256;                 // tokens per tile (MMA N)
 constexpr int kBK = 64;                  // k per stage (one 128-byte swizzle atom of bf16)
-constexpr int kStages = 3;
+constexpr int kXStages = 3;              // X tiles in flight (TMA)
+constexpr int kWStages = 4;              // dequantised weight tiles in flight (decode warps)
 constexpr int kCodeRing = 7;             // code stages in flight per decode thread
 constexpr int kDecodeWarps = 8;
 constexpr int kDecodeThreads = 32 * kDecodeWarps;  // two threads per weight row
@@ -127,6 +128,19 @@ __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, vola
 {
     if (mbar_try_wait(bar, parity)) return true;
     return wait_slow(bar, parity, abort_flag, ws, who, drain);
+}
+
+// One lane of the warp, chosen by the hardware; the rest of the warp keeps the
+// same (uniform) control flow and operands.
+__device__ __forceinline__ bool elect_one()
+{
+    uint32_t pred;
+    asm volatile(
+        "{\n\t.reg .pred P;\n\t.reg .b32 R;\n\t"
+        "elect.sync R|P, 0xffffffff;\n\t"
+        "selp.u32 %0, 1, 0, P;\n\t}"
+        : "=r"(pred));
+    return pred != 0;
 }
 
 // One lane of the warp polls (a barrier polled by many threads serialises);
@@ -257,12 +271,12 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
     const uint32_t sbase = smem_u32(smem_raw);
     const uint32_t tab = (sbase + 32767u) & ~32767u;
     const uint32_t xs0 = tab + kTabBytes4;
-    const uint32_t ws0 = xs0 + kStages * kXStageBytes;
+    const uint32_t ws0 = xs0 + kXStages * kXStageBytes;
     constexpr uint32_t kLowBytes = kCodeRing * kCodeStageBytes + 256;
     const bool low = tab - sbase >= kLowBytes;
-    const uint32_t cr0 = low ? sbase : ws0 + kStages * kWStageBytes;
+    const uint32_t cr0 = low ? sbase : ws0 + kWStages * kWStageBytes;
     const uint32_t bar0 = cr0 + kCodeRing * kCodeStageBytes;
-    const uint32_t layout_end = low ? ws0 + kStages * kWStageBytes : bar0 + 256;
+    const uint32_t layout_end = low ? ws0 + kWStages * kWStageBytes : bar0 + 256;
     if (layout_end > sbase + p.smem_bytes) {          // launch too small for this layout: refuse
         if (threadIdx.x == 0) {
             atomicExch(&p.ws->detail, (uint32_t)kWaitLayout);
@@ -271,22 +285,28 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         return;
     }
     uint8_t* gen = smem_raw - sbase;                  // generic pointer = gen + shared address
-    // barriers: xfull[S], wfull[S], empty[S], accfull[2], accempty[2], then tmem slot and abort flag
+    // barriers: xfull[X], xempty[X], wfull[W], wempty[W], accfull[2], accempty[2], drain,
+    // then the tmem slot and the abort flag
     auto xfull = [&](int s) { return bar0 + 8u * s; };
-    auto wfull = [&](int s) { return bar0 + 8u * (kStages + s); };
-    auto empty = [&](int s) { return bar0 + 8u * (2 * kStages + s); };
-    auto accfull = [&](int b) { return bar0 + 8u * (3 * kStages + b); };
-    auto accempty = [&](int b) { return bar0 + 8u * (3 * kStages + 2 + b); };
-    const uint32_t drainb = bar0 + 8u * (3 * kStages + 4);
-    const uint32_t tmem_slot = bar0 + 8u * (3 * kStages + 5);
+    auto xempty = [&](int s) { return bar0 + 8u * (kXStages + s); };
+    auto wfull = [&](int s) { return bar0 + 8u * (2 * kXStages + s); };
+    auto wempty = [&](int s) { return bar0 + 8u * (2 * kXStages + kWStages + s); };
+    constexpr int kB0 = 2 * kXStages + 2 * kWStages;
+    auto accfull = [&](int b) { return bar0 + 8u * (kB0 + b); };
+    auto accempty = [&](int b) { return bar0 + 8u * (kB0 + 2 + b); };
+    const uint32_t drainb = bar0 + 8u * (kB0 + 4);
+    const uint32_t tmem_slot = bar0 + 8u * (kB0 + 5);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(gen + tmem_slot + 8);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     if (tid == 0) {
-        for (int s = 0; s < kStages; ++s) {
+        for (int s = 0; s < kXStages; ++s) {
             mbar_init(xfull(s), 1);
+            mbar_init(xempty(s), 1);
+        }
+        for (int s = 0; s < kWStages; ++s) {
             mbar_init(wfull(s), kDecodeWarps);
-            mbar_init(empty(s), 1);
+            mbar_init(wempty(s), 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(accfull(b), 1);
@@ -324,77 +344,89 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
 
     if (warp == 0) {
         // ---------------- TMA producer ----------------
-        if (lane == 0) {
-            int stage = 0;
-            uint32_t phase = 0;
-            bool ok = true;
-            uint32_t issued = 0, issued_par = 0;       // per stage: used at least once / parity of last load
-            // the code rows of a tile are one contiguous block: ask L2 for it one
-            // tile ahead so the decode warps' copies hit L2
-            auto prefetch_codes = [&](int tile) {
-                if (tile >= ntiles) return;
-                const int64_t n0 = (int64_t)(tile % p.n_tiles_n) * kBM;
-                const int64_t rows = (p.N - n0) < kBM ? (p.N - n0) : kBM;
-                const uint8_t* base = p.codes + n0 * p.row_bytes;
-                const int64_t bytes = rows * p.row_bytes;
-                for (int64_t off = 0; off < bytes; off += 16384) {
-                    const int64_t nb = (bytes - off) < 16384 ? (bytes - off) : 16384;
-                    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base + off), "r"((uint32_t)nb)
-                                 : "memory");
+        // The whole warp walks the loop (uniform operands); one elected lane issues.
+        int stage = 0;
+        uint32_t phase = 0;
+        bool ok = true;
+        uint32_t issued = 0, issued_par = 0;           // per stage: used at least once / parity of last load
+        // the code rows of a tile are one contiguous block: ask L2 for it one
+        // tile ahead so the decode warps' copies hit L2
+        auto prefetch_codes = [&](int tile) {
+            if (tile >= ntiles) return;
+            const int64_t n0 = (int64_t)(tile % p.n_tiles_n) * kBM;
+            const int64_t rows = (p.N - n0) < kBM ? (p.N - n0) : kBM;
+            const uint8_t* base = p.codes + n0 * p.row_bytes;
+            const int64_t bytes = rows * p.row_bytes;
+            for (int64_t off = (int64_t)lane * 16384; off < bytes; off += 32 * 16384) {
+                const int64_t nb = (bytes - off) < 16384 ? (bytes - off) : 16384;
+                asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base + off), "r"((uint32_t)nb)
+                             : "memory");
+            }
+        };
+        prefetch_codes(blockIdx.x);
+        for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+            const int t0 = (tile / p.n_tiles_n) * kBN;
+            prefetch_codes(tile + gridDim.x);
+            for (int ks = 0; ks < ksteps; ++ks) {
+                if (!warp_wait(xempty(stage), phase ^ 1u, abort_flag, p.ws, kWaitProducer)) {
+                    ok = false;
+                    break;
                 }
-            };
-            prefetch_codes(blockIdx.x);
-            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
-                const int t0 = (tile / p.n_tiles_n) * kBN;
-                prefetch_codes(tile + gridDim.x);
-                for (int ks = 0; ks < ksteps; ++ks) {
-                    if (!wait_bounded(empty(stage), phase ^ 1u, abort_flag, p.ws, kWaitProducer)) {
-                        ok = false;
-                        break;
-                    }
+                if (elect_one()) {
                     mbar_expect_tx(xfull(stage), kXStageBytes);
                     tma_load_2d(xs0 + stage * kXStageBytes, &xmap, ks * kBK, t0, xfull(stage));
-                    issued |= 1u << stage;
-                    issued_par = (issued_par & ~(1u << stage)) | (phase << stage);
-                    if (++stage == kStages) { stage = 0; phase ^= 1u; }
                 }
+                __syncwarp();
+                issued |= 1u << stage;
+                issued_par = (issued_par & ~(1u << stage)) | (phase << stage);
+                if (++stage == kXStages) { stage = 0; phase ^= 1u; }
             }
-            // every load this thread issued has landed before the CTA can leave
-            for (int st = 0; st < kStages; ++st)
+        }
+        // every load this warp issued has landed before the CTA can leave
+        if (lane == 0)
+            for (int st = 0; st < kXStages; ++st)
                 if (issued & (1u << st))
                     wait_bounded(xfull(st), (issued_par >> st) & 1u, abort_flag, p.ws, kWaitDrain, true);
-        }
+        __syncwarp();
     } else if (warp == 1) {
         // ---------------- MMA issuer ----------------
-        if (lane == 0) {
-            int stage = 0;
-            uint32_t phase = 0;
-            bool ok = true;
-            int it = 0;
-            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
-                const int buf = it & 1;
-                const uint32_t acc_phase = ((uint32_t)it >> 1) & 1u;
-                if (!wait_bounded(accempty(buf), acc_phase ^ 1u, abort_flag, p.ws, kWaitMma)) break;
+        // The whole warp walks the loop, so descriptors and addresses stay
+        // warp-uniform; one elected lane issues the MMAs and commits.
+        int xs = 0, wsg = 0;
+        uint32_t xph = 0, wph = 0;
+        bool ok = true;
+        int it = 0;
+        for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
+            const int buf = it & 1;
+            const uint32_t acc_phase = ((uint32_t)it >> 1) & 1u;
+            if (!warp_wait(accempty(buf), acc_phase ^ 1u, abort_flag, p.ws, kWaitMma)) break;
+            tc_fence_after();
+            const uint32_t dcol = tmem_base + (uint32_t)(buf * kBN);
+            for (int ks = 0; ks < ksteps; ++ks) {
+                if (!warp_wait(xfull(xs), xph, abort_flag, p.ws, kWaitMma) ||
+                    !warp_wait(wfull(wsg), wph, abort_flag, p.ws, kWaitMma)) {
+                    ok = false;
+                    break;
+                }
                 tc_fence_after();
-                const uint32_t dcol = tmem_base + (uint32_t)(buf * kBN);
-                for (int ks = 0; ks < ksteps; ++ks) {
-                    if (!wait_bounded(xfull(stage), phase, abort_flag, p.ws, kWaitMma) ||
-                        !wait_bounded(wfull(stage), phase, abort_flag, p.ws, kWaitMma)) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    const uint64_t adesc = smem_desc_sw128(ws0 + stage * kWStageBytes);
-                    const uint64_t bdesc = smem_desc_sw128(xs0 + stage * kXStageBytes);
+                const uint64_t adesc = smem_desc_sw128(ws0 + wsg * kWStageBytes);
+                const uint64_t bdesc = smem_desc_sw128(xs0 + xs * kXStageBytes);
+                if (elect_one()) {
 #pragma unroll
                     for (int kk = 0; kk < kBK / 16; ++kk) {
                         // 16 k of bf16 = 32 bytes (2 descriptor units) further inside the swizzle atom
                         mma_f16(dcol, adesc + 2 * kk, bdesc + 2 * kk, p.idesc, (ks | kk) != 0);
                     }
-                    mma_commit(empty(stage));
-                    if (++stage == kStages) { stage = 0; phase ^= 1u; }
+                    mma_commit(xempty(xs));
+                    mma_commit(wempty(wsg));
                 }
-                if (ok) mma_commit(accfull(buf));
+                __syncwarp();
+                if (++xs == kXStages) { xs = 0; xph ^= 1u; }
+                if (++wsg == kWStages) { wsg = 0; wph ^= 1u; }
+            }
+            if (ok) {
+                if (elect_one()) mma_commit(accfull(buf));
+                __syncwarp();
             }
         }
     } else if (warp >= 2 && warp < 6) {
@@ -471,34 +503,23 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
             if (g < total) step(ahead);
             cp_async_commit();
         };
-        for (int g = 0; g < kCodeRing - 1; ++g) issue(g);
-        int slot = 0;                                   // g % kCodeRing
-        for (int g = 0; g < total; ++g) {
-            issue(g + kCodeRing - 1);
-            cp_async_wait<kCodeRing - 1>();
-            const bool valid = cur.valid;
+        // Resolve the codes of one stage (its slot in the ring) into 16 pair values.
+        auto resolve = [&](int slot, bool valid, uint32_t (&pr)[16]) {
             uint4 cv = make_uint4(0, 0, 0, 0);
             if (valid) cv = lds128(cr0 + slot * kCodeStageBytes + d * kCodeSlotBytes);
-            if (++slot == kCodeRing) slot = 0;
-            step(cur);
             const uint32_t cw[4] = {cv.x, cv.y, cv.z, cv.w};
-            if (!warp_wait(empty(stage), phase ^ 1u, abort_flag, p.ws, kWaitDecode)) break;
-            const uint32_t wrow = ws0 + stage * kWStageBytes + r * 128;
-            const uint32_t sw = (uint32_t)(r & 7);
             if (p.bits == 4) {
                 // word i holds k = 32h + 8i .. +7 -> 16-byte chunk 4h + i of the row
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                     const uint32_t c = cw[i];
-                    const uint32_t a0 = lds32(((c << 7) & 0x7f80u) | tl);
-                    const uint32_t a1 = lds32(((c >> 1) & 0x7f80u) | tl);
-                    const uint32_t a2 = lds32(((c >> 9) & 0x7f80u) | tl);
-                    const uint32_t a3 = lds32(((c >> 17) & 0x7f80u) | tl);
-                    sts128(wrow + ((((uint32_t)(4 * h + i)) ^ sw) << 4), a0, a1, a2, a3);
+                    pr[4 * i + 0] = lds32(((c << 7) & 0x7f80u) | tl);
+                    pr[4 * i + 1] = lds32(((c >> 1) & 0x7f80u) | tl);
+                    pr[4 * i + 2] = lds32(((c >> 9) & 0x7f80u) | tl);
+                    pr[4 * i + 3] = lds32(((c >> 17) & 0x7f80u) | tl);
                 }
             } else {
                 // one 12-byte group of 32 k; pair p -> chunk 4h + p / 4
-                uint32_t pr[16];
 #pragma unroll
                 for (int i = 0; i < 3; ++i) {
                     pr[5 * i + 0] = lds32(((cw[i] << 7) & 0x1f80u) | tl);
@@ -508,15 +529,40 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
                     pr[5 * i + 4] = lds32(((cw[i] >> 17) & 0x1f80u) | tl);
                 }
                 pr[15] = lds32(((cw[0] >> 23) & 0x0180u) | ((cw[1] >> 21) & 0x0600u) | ((cw[2] >> 19) & 0x1800u) | tl);
-#pragma unroll
-                for (int i = 0; i < 4; ++i)
-                    sts128(wrow + ((((uint32_t)(4 * h + i)) ^ sw) << 4), pr[4 * i], pr[4 * i + 1], pr[4 * i + 2],
-                           pr[4 * i + 3]);
             }
+        };
+        // Software pipeline: the pairs of stage g+1 are looked up while stage g
+        // waits for its weight slot and is stored.
+        for (int g = 0; g < kCodeRing - 1; ++g) issue(g);
+        uint32_t cur_pr[16], next_pr[16];
+        int slot = 0;                                   // ring slot of stage g
+        if (total > 0) {
+            issue(kCodeRing - 1);
+            cp_async_wait<kCodeRing - 1>();
+            resolve(slot, cur.valid, cur_pr);
+            step(cur);
+        }
+        for (int g = 0; g < total; ++g) {
+            if (++slot == kCodeRing) slot = 0;
+            if (g + 1 < total) {
+                issue(g + kCodeRing);
+                cp_async_wait<kCodeRing - 1>();
+                resolve(slot, cur.valid, next_pr);
+                step(cur);
+            }
+            if (!warp_wait(wempty(stage), phase ^ 1u, abort_flag, p.ws, kWaitDecode)) break;
+            const uint32_t wrow = ws0 + stage * kWStageBytes + r * 128;
+            const uint32_t sw = (uint32_t)(r & 7);
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                sts128(wrow + ((((uint32_t)(4 * h + i)) ^ sw) << 4), cur_pr[4 * i], cur_pr[4 * i + 1],
+                       cur_pr[4 * i + 2], cur_pr[4 * i + 3]);
             fence_proxy_async();          // this thread's tile writes -> visible to the tensor core
             __syncwarp();
             if (lane == 0) mbar_arrive(wfull(stage));
-            if (++stage == kStages) { stage = 0; phase ^= 1u; }
+            if (++stage == kWStages) { stage = 0; phase ^= 1u; }
+#pragma unroll
+            for (int i = 0; i < 16; ++i) cur_pr[i] = next_pr[i];
         }
         cp_async_wait<0>();
     }
@@ -524,7 +570,7 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
     // teardown: every MMA this CTA issued has completed before TMEM is freed
     __syncthreads();
     if (warp == 1) {
-        if (lane == 0) {
+        if (elect_one()) {
             mma_commit(drainb);
             wait_bounded(drainb, 0, abort_flag, p.ws, kWaitDrain, true);
         }
@@ -565,7 +611,7 @@ uint32_t make_idesc(bool f16_inputs)
     return d;
 }
 
-constexpr uint32_t kStageRegion = kStages * (kXStageBytes + kWStageBytes);
+constexpr uint32_t kStageRegion = kXStages * kXStageBytes + kWStages * kWStageBytes;
 constexpr uint32_t kRingRegion = kCodeRing * kCodeStageBytes + 256;
 
 // Dynamic shared memory for the layout above, given where the dynamic region
