@@ -176,6 +176,33 @@ logq_status logq_quantize_noalloc(const float* W, int64_t N, int64_t K, int bits
                                   double range, int flags, uint8_t* codes,
                                   logq_codebook* cb_out, void* stream);
 
+/* One matrix of logq_linear_grouped. */
+typedef struct logq_linear_item {
+    const uint8_t* codes;       /* device: packed codes of this matrix, N rows */
+    const logq_codebook* cb;    /* host: its codebook */
+    int64_t N;                  /* rows of the matrix = outputs per batch row */
+    void* Y;                    /* device: output [B][N] in y_dtype */
+} logq_linear_item;
+
+/*
+ * Several quantised linear layers that read the same activations X[B][K] --
+ * e.g. the q/k/v or the gate/up projections of a transformer layer -- each
+ * with its own per-tensor codebook (Sec. 3.1) and output: Y_i = X * What_i^T
+ * (Sec. 3.3), in one call.  count is 1..4 and all items share the code width
+ * of their codebooks.  With B <= 16 (4-bit) or B <= 4 (3-bit) the matrices
+ * share a single decode-GEMV launch; larger B runs one prefill launch each.
+ * l2_prefetch (device, may be NULL) / l2_prefetch_bytes name a range the
+ * call asks the L2 cache to fetch while it runs -- for a decode step, the
+ * codes of the next layer -- a hint only: it is never read by the
+ * computation and may be any readable device memory.  Asynchronous; errors
+ * as logq_linear (LOGQ_ERR_INVALID_ARG also for count outside 1..4 or items
+ * of different code widths).
+ */
+logq_status logq_linear_grouped(const logq_linear_item* items, int count, const void* X,
+                                logq_dtype x_dtype, int64_t B, int64_t K, logq_dtype y_dtype,
+                                const void* l2_prefetch, size_t l2_prefetch_bytes,
+                                void* workspace, size_t workspace_bytes, void* stream);
+
 /* Synchronise `stream`, read the device error word of `workspace`, clear it,
  * and return LOGQ_OK or LOGQ_ERR_TIMEOUT.  *detail (host, may be NULL)
  * receives an implementation code naming the wait that gave up. */

@@ -38,7 +38,7 @@ LOGQ_SHIFT_EXACT, LOGQ_SHIFT_FLOOR = 0, 1
 
 EXPORTED = ("logq_build_codebook", "logq_packed_bytes", "logq_workspace_bytes", "logq_quantize",
             "logq_linear", "logq_workspace_status", "logq_status_string", "logq_device_sm_count",
-            "logq_quantize_noalloc")
+            "logq_quantize_noalloc", "logq_linear_grouped")
 
 
 class Codebook(ctypes.Structure):
@@ -55,6 +55,16 @@ class Codebook(ctypes.Structure):
         ("thresh", ctypes.c_float * 8),
         ("level_bf16", ctypes.c_uint16 * 16),
         ("level_f16", ctypes.c_uint16 * 16),
+    ]
+
+
+class LinearItem(ctypes.Structure):
+    """Mirror of ``logq_linear_item`` (include/logq.h)."""
+    _fields_ = [
+        ("codes", ctypes.c_void_p),
+        ("cb", ctypes.POINTER(Codebook)),
+        ("N", ctypes.c_int64),
+        ("Y", ctypes.c_void_p),
     ]
 
 
@@ -84,6 +94,9 @@ def _load() -> ctypes.CDLL:
     lib.logq_linear.argtypes = [P, ctypes.POINTER(Codebook), P, c_int, c_i64, c_i64, c_i64, P,
                                 c_int, P, ctypes.c_size_t, P]
     lib.logq_linear.restype = c_int
+    lib.logq_linear_grouped.argtypes = [ctypes.POINTER(LinearItem), c_int, P, c_int, c_i64, c_i64, c_int,
+                                        P, ctypes.c_size_t, P, ctypes.c_size_t, P]
+    lib.logq_linear_grouped.restype = c_int
     lib.logq_workspace_status.argtypes = [P, P, ctypes.POINTER(ctypes.c_uint32)]
     lib.logq_workspace_status.restype = c_int
     lib.logq_status_string.argtypes = [c_int]
@@ -212,6 +225,37 @@ def logq_linear(codes, cb: Codebook, X, N: int, K: int, y_dtype=None, Y=None, wo
                          ctypes.c_void_p(workspace.data_ptr()), workspace.numel(), _stream_ptr(stream))
     _check(st, "logq_linear")
     return Y
+
+
+def logq_linear_grouped(items, X, K: int, y_dtype=None, workspace=None, prefetch=None,
+                        prefetch_bytes: int = 0, stream=None):
+    """One launch for up to four matrices sharing X: items = [(codes, cb, N, Y or None), ...].
+    prefetch: optional device tensor (or (tensor, bytes)) the call warms L2 with.
+    Returns the list of outputs."""
+    import torch
+    assert X.is_cuda and X.dim() == 2 and X.is_contiguous() and X.shape[1] == K
+    B = X.shape[0]
+    xd = _dtype_code(X.dtype)
+    yd = LOGQ_F32 if y_dtype is None else (_dtype_code(y_dtype) if not isinstance(y_dtype, int) else y_dtype)
+    arr = (LinearItem * len(items))()
+    outs = []
+    keep = []
+    for i, (codes, cb, N, Y) in enumerate(items):
+        if Y is None:
+            Y = torch.empty((B, N), dtype=_torch_dtype(yd), device=X.device)
+        outs.append(Y)
+        keep.append(cb)
+        arr[i] = LinearItem(ctypes.c_void_p(codes.data_ptr()), ctypes.pointer(cb), int(N),
+                            ctypes.c_void_p(Y.data_ptr()))
+    if workspace is None:
+        workspace = new_workspace(X.device)
+    pf_ptr = ctypes.c_void_p(prefetch.data_ptr()) if prefetch is not None else None
+    pf_bytes = int(prefetch_bytes) if prefetch is not None else 0
+    st = _lib().logq_linear_grouped(arr, len(items), ctypes.c_void_p(X.data_ptr()), xd, B, int(K), yd, pf_ptr,
+                                    pf_bytes, ctypes.c_void_p(workspace.data_ptr()), workspace.numel(),
+                                    _stream_ptr(stream))
+    _check(st, "logq_linear_grouped")
+    return outs
 
 
 def logq_workspace_status(workspace, stream=None):

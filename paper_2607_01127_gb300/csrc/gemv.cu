@@ -22,6 +22,7 @@
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <stdint.h>
+#include <string.h>
 
 #include "internal.h"
 
@@ -40,20 +41,35 @@ constexpr int64_t kPrefetchCap = 1 << 20;     // bytes of codes prefetched per C
 // table (64 KiB at 4 bits) + up to 64 KiB of alignment pad + span partials
 constexpr int kMaxSmem = 65536 + 256 * kTabStride + kRedBytes;
 
-struct GemvParams {
+constexpr int kMaxItems = 4;
+
+// One matrix of a grouped launch: all items share X, K, B and the code width.
+struct GemvItem {
     const uint8_t* codes;
-    const uint16_t* X;
     void* Y;
-    int64_t N;
+    int32_t N;
+    int32_t cta_begin;    // first CTA of this item
+    int32_t cta_count;    // CTAs assigned to it
+    int32_t rows_q;       // N / cta_count
+    int32_t rows_rem;     // N % cta_count (the first rows_rem CTAs take one more row)
+    int32_t _pad;
+    uint32_t lvl16[16];   // code-indexed 16-bit levels (low half used)
+};
+
+struct GemvParams {
+    GemvItem item[kMaxItems];
+    int32_t nitems;
     int32_t K;
     int32_t B;
+    int32_t y_dtype;
+    const uint16_t* X;
     int64_t row_bytes;
     int32_t spans;        // S: spans of 32*KW k covering K
     int32_t groups;       // G: warps sharing one span (row-parallel)
     int32_t span_cols;    // warps / G: spans in flight at once
     int32_t chunk_rows;   // rows reduced per shared-memory pass
-    int32_t y_dtype;
-    uint32_t lvl16[16];   // code-indexed 16-bit levels (low half used)
+    const uint8_t* pf;    // optional L2 warm-up range (e.g. the next layer's codes)
+    int64_t pf_bytes;
 };
 
 __device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel)
@@ -242,20 +258,37 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
     static_assert(V <= 32 && (V & (V - 1)) == 0, "values per lane must be a power of two <= 32");
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int64_t C = gridDim.x;
-    const int64_t r0 = (p.N * (int64_t)blockIdx.x) / C;
-    const int64_t r1 = (p.N * ((int64_t)blockIdx.x + 1)) / C;
+    // this CTA's matrix and its contiguous range of rows
+    int m = 0;
+#pragma unroll
+    for (int i = 1; i < kMaxItems; ++i)
+        if (i < p.nitems && (int)blockIdx.x >= p.item[i].cta_begin) m = i;
+    const GemvItem& item = p.item[m];
+    const int c = (int)blockIdx.x - item.cta_begin;
+    const int64_t r0 = (int64_t)c * item.rows_q + (c < item.rows_rem ? c : item.rows_rem);
+    const int64_t r1 = r0 + item.rows_q + (c < item.rows_rem ? 1 : 0);
 
-    // 1) start streaming this CTA's code rows into L2.
+    // 1) start streaming this CTA's code rows into L2, and its share of the
+    //    optional warm-up range.
     {
-        const uint8_t* base = p.codes + r0 * p.row_bytes;
+        constexpr int64_t piece = 16384;
+        const uint8_t* base = item.codes + r0 * p.row_bytes;
         int64_t bytes = (r1 - r0) * p.row_bytes;
         if (bytes > kPrefetchCap) bytes = kPrefetchCap;
-        constexpr int64_t piece = 16384;
         for (int64_t off = (int64_t)tid * piece; off < bytes; off += (int64_t)kThreads * piece) {
             const int64_t n = (bytes - off) < piece ? (bytes - off) : piece;
             asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base + off), "r"((uint32_t)n)
                          : "memory");
+        }
+        if (p.pf_bytes > 0) {
+            const int64_t share = ((p.pf_bytes + gridDim.x - 1) / gridDim.x + 15) & ~(int64_t)15;
+            const int64_t beg = share * blockIdx.x;
+            const int64_t end = (beg + share < p.pf_bytes) ? beg + share : p.pf_bytes;
+            for (int64_t off = beg + (int64_t)tid * piece; off < end; off += (int64_t)kThreads * piece) {
+                const int64_t n = (end - off) < piece ? (end - off) : piece;
+                asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p.pf + off), "r"((uint32_t)n)
+                             : "memory");
+            }
         }
     }
 
@@ -273,7 +306,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
         const int e = i >> 3, part = i & 7;
         const uint32_t lo = (BITS == 4) ? (e & 15) : (e & 7);
         const uint32_t hi = (BITS == 4) ? (e >> 4) : (e >> 3);
-        const uint32_t v = (p.lvl16[lo] & 0xffffu) | (p.lvl16[hi] << 16);
+        const uint32_t v = (item.lvl16[lo] & 0xffffu) | (item.lvl16[hi] << 16);
         reinterpret_cast<uint4*>(tab + e * (kTabStride / 4))[part] = make_uint4(v, v, v, v);
     }
     __syncthreads();
@@ -319,7 +352,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                 }
                 // idle lanes read the row start (valid memory) and multiply by zero
                 const int64_t lane_byte = active ? ((BITS == 4) ? (int64_t)k0 / 2 : (int64_t)k0 / 32 * 12) : 0;
-                const uint8_t* first = p.codes + (q0 + g) * p.row_bytes + lane_byte;
+                const uint8_t* first = item.codes + (q0 + g) * p.row_bytes + lane_byte;
 
                 // Rounds of R rows with two code buffers: the loads of round t+1 are
                 // in flight while round t is decoded.  Full rounds run unguarded;
@@ -371,7 +404,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
             if (b >= p.B) continue;
             float sum = 0.f;
             for (int s = 0; s < p.spans; ++s) sum += red[((int64_t)s * p.chunk_rows + lr) * B + b];
-            store_y(p.Y, p.y_dtype, (int64_t)b * p.N + q0 + lr, sum);
+            store_y(item.Y, p.y_dtype, (int64_t)b * item.N + q0 + lr, sum);
         }
         __syncthreads();
     }
@@ -455,18 +488,19 @@ bool gemv_supports(int bits, int64_t B)
     return false;
 }
 
-cudaError_t launch_gemv(const LinearArgs& a, cudaStream_t s)
+cudaError_t launch_gemv_group(const GroupArgs& a, cudaStream_t s)
 {
+    if (a.count < 1 || a.count > kMaxItems) return cudaErrorInvalidValue;
     const int Bp = padded_batch(a.B);
     const int KW = kw_for(a.bits, Bp);
     const int span = 32 * KW;
     GemvParams p;
-    p.codes = a.codes;
+    memset(&p, 0, sizeof p);
+    p.nitems = a.count;
     p.X = static_cast<const uint16_t*>(a.X);
-    p.Y = a.Y;
-    p.N = a.N;
     p.K = (int32_t)a.K;
     p.B = (int32_t)a.B;
+    p.y_dtype = a.y_dtype;
     p.row_bytes = (a.bits == 4) ? a.K / 2 : a.K / 32 * 12;
     p.spans = (int32_t)((a.K + span - 1) / span);
     if (p.spans >= kWarps) {
@@ -476,19 +510,92 @@ cudaError_t launch_gemv(const LinearArgs& a, cudaStream_t s)
         p.groups = kWarps / p.spans;
         p.span_cols = p.spans;
     }
+    p.pf = static_cast<const uint8_t*>(a.pf);
+    p.pf_bytes = a.pf ? a.pf_bytes : 0;
+
+    // CTAs in proportion to each matrix's rows (at least one each, at most one per row).
     const int sms = sm_count() > 0 ? sm_count() : 148;
-    const int64_t grid = a.N < sms ? a.N : sms;
-    const int64_t rows_per_cta = (a.N + grid - 1) / grid;
+    int64_t total_rows = 0;
+    for (int i = 0; i < a.count; ++i) total_rows += a.item[i].N;
+    int grid = (int)(total_rows < sms ? total_rows : sms);
+    if (grid < a.count) grid = a.count;
+    int ctas[kMaxItems] = {0};
+    int used = 0;
+    for (int i = 0; i < a.count; ++i) {
+        int64_t c = (int64_t)grid * a.item[i].N / total_rows;
+        if (c < 1) c = 1;
+        if (c > a.item[i].N) c = a.item[i].N;
+        ctas[i] = (int)c;
+        used += ctas[i];
+    }
+    while (used < grid) {               // hand out what rounding left, largest rows per CTA first
+        int best = -1;
+        double best_load = -1.0;
+        for (int i = 0; i < a.count; ++i) {
+            if (ctas[i] >= a.item[i].N) continue;
+            const double load = (double)a.item[i].N / ctas[i];
+            if (load > best_load) { best_load = load; best = i; }
+        }
+        if (best < 0) break;
+        ++ctas[best];
+        ++used;
+    }
+    while (used > grid) {               // too many (minimums): take from the lightest
+        int best = -1;
+        double best_load = 1e300;
+        for (int i = 0; i < a.count; ++i) {
+            if (ctas[i] <= 1) continue;
+            const double load = (double)a.item[i].N / ctas[i];
+            if (load < best_load) { best_load = load; best = i; }
+        }
+        if (best < 0) break;
+        --ctas[best];
+        --used;
+    }
+    grid = used;
+    int64_t max_rows = 0;
+    int begin = 0;
+    for (int i = 0; i < a.count; ++i) {
+        GemvItem& it = p.item[i];
+        it.codes = a.item[i].codes;
+        it.Y = a.item[i].Y;
+        it.N = (int32_t)a.item[i].N;
+        it.cta_begin = begin;
+        it.cta_count = ctas[i];
+        it.rows_q = (int32_t)(a.item[i].N / ctas[i]);
+        it.rows_rem = (int32_t)(a.item[i].N % ctas[i]);
+        for (int c = 0; c < 16; ++c) it.lvl16[c] = a.item[i].lvl16[c];
+        begin += ctas[i];
+        const int64_t rows = it.rows_q + (it.rows_rem ? 1 : 0);
+        if (rows > max_rows) max_rows = rows;
+    }
     int64_t chunk = kRedBytes / ((int64_t)p.spans * Bp * 4);
-    if (chunk > rows_per_cta) chunk = rows_per_cta;
+    if (chunk > max_rows) chunk = max_rows;
     if (chunk < 1) return cudaErrorInvalidValue;
     p.chunk_rows = (int32_t)chunk;
-    p.y_dtype = a.y_dtype;
-    for (int c = 0; c < 16; ++c) p.lvl16[c] = a.lvl16[c];
     const int nent = (a.bits == 4) ? 256 : 64;
     const size_t smem = 65536 + (size_t)nent * kTabStride + (size_t)p.spans * chunk * Bp * 4;
-    return a.x_f16 ? dispatch<true>(a.bits, Bp, p, (int)grid, smem, s)
-                   : dispatch<false>(a.bits, Bp, p, (int)grid, smem, s);
+    return a.x_f16 ? dispatch<true>(a.bits, Bp, p, grid, smem, s)
+                   : dispatch<false>(a.bits, Bp, p, grid, smem, s);
+}
+
+cudaError_t launch_gemv(const LinearArgs& a, cudaStream_t s)
+{
+    GroupArgs g;
+    memset(&g, 0, sizeof g);
+    g.count = 1;
+    g.item[0].codes = a.codes;
+    g.item[0].Y = a.Y;
+    g.item[0].N = a.N;
+    for (int c = 0; c < 16; ++c) g.item[0].lvl16[c] = a.lvl16[c];
+    g.X = a.X;
+    g.B = a.B;
+    g.K = a.K;
+    g.bits = a.bits;
+    g.x_f16 = a.x_f16;
+    g.y_dtype = a.y_dtype;
+    g.ws = a.ws;
+    return launch_gemv_group(g, s);
 }
 
 }  // namespace logq

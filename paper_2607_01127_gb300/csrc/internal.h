@@ -41,11 +41,34 @@ struct LinearArgs {
     Workspace* ws;
 };
 
+// A grouped decode launch: up to four matrices that share X (e.g. q/k/v or
+// gate/up), each with its own codebook and output.
+struct GroupItem {
+    const uint8_t* codes;
+    void* Y;
+    int64_t N;
+    uint16_t lvl16[16];
+};
+
+struct GroupArgs {
+    GroupItem item[4];
+    int count;
+    const void* X;
+    int64_t B, K;
+    int bits;
+    int x_f16;
+    int y_dtype;
+    const void* pf;          // optional L2 warm-up range
+    int64_t pf_bytes;
+    Workspace* ws;
+};
+
 int sm_count();
 cudaError_t launch_absmax(const float* W, int64_t count, Workspace* ws, cudaStream_t s);
 cudaError_t launch_quantize(const float* W, int64_t N, int64_t K, const QuantParams& p,
                             uint8_t* codes, Workspace* ws, cudaStream_t s);
 cudaError_t launch_gemv(const LinearArgs& a, cudaStream_t s);
+cudaError_t launch_gemv_group(const GroupArgs& a, cudaStream_t s);
 cudaError_t launch_prefill(const LinearArgs& a, cudaStream_t s);
 bool gemv_supports(int bits, int64_t B);
 

@@ -233,6 +233,59 @@ logq_status logq_linear(const uint8_t* codes, const logq_codebook* cb, const voi
     return cuda_status(e);
 }
 
+logq_status logq_linear_grouped(const logq_linear_item* items, int count, const void* X,
+                                logq_dtype x_dtype, int64_t B, int64_t K, logq_dtype y_dtype,
+                                const void* l2_prefetch, size_t l2_prefetch_bytes,
+                                void* workspace, size_t workspace_bytes, void* stream)
+{
+    if (!items || count < 1 || count > 4 || !X || !aligned16(X)) return LOGQ_ERR_INVALID_ARG;
+    if (x_dtype != LOGQ_BF16 && x_dtype != LOGQ_F16) return LOGQ_ERR_UNSUPPORTED;
+    if (y_dtype != LOGQ_F32 && y_dtype != x_dtype) return LOGQ_ERR_UNSUPPORTED;
+    if (B <= 0 || B > (int64_t(1) << 31) || K > (int64_t(1) << 30)) return LOGQ_ERR_INVALID_ARG;
+    if (!workspace || !aligned16(workspace) || workspace_bytes < kWorkspaceBytes) return LOGQ_ERR_WORKSPACE;
+    if (l2_prefetch_bytes > 0 && !l2_prefetch) return LOGQ_ERR_INVALID_ARG;
+    int bits = 0;
+    for (int i = 0; i < count; ++i) {
+        const logq_linear_item& it = items[i];
+        if (!it.codes || !it.cb || !it.Y || !aligned16(it.codes) || !aligned16(it.Y)) return LOGQ_ERR_INVALID_ARG;
+        if (it.N > (int64_t(1) << 31) || logq_packed_bytes(it.N, K, it.cb->bits) == 0) return LOGQ_ERR_INVALID_ARG;
+        if (it.cb->qmax != (1 << (it.cb->bits - 1)) - 1) return LOGQ_ERR_INVALID_ARG;
+        if (i == 0) bits = it.cb->bits;
+        else if (it.cb->bits != bits) return LOGQ_ERR_INVALID_ARG;
+    }
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    Workspace* ws = static_cast<Workspace*>(workspace);
+    const int x_f16 = (x_dtype == LOGQ_F16);
+    if (gemv_supports(bits, B)) {
+        GroupArgs g;
+        memset(&g, 0, sizeof g);
+        g.count = count;
+        for (int i = 0; i < count; ++i) {
+            g.item[i].codes = items[i].codes;
+            g.item[i].Y = items[i].Y;
+            g.item[i].N = items[i].N;
+            const uint16_t* tab = x_f16 ? items[i].cb->level_f16 : items[i].cb->level_bf16;
+            for (int c = 0; c < (1 << bits); ++c) g.item[i].lvl16[c] = tab[c];
+        }
+        g.X = X;
+        g.B = B;
+        g.K = K;
+        g.bits = bits;
+        g.x_f16 = x_f16;
+        g.y_dtype = (int)y_dtype;
+        g.pf = l2_prefetch;
+        g.pf_bytes = (int64_t)((l2_prefetch_bytes / 16) * 16);
+        g.ws = ws;
+        return cuda_status(launch_gemv_group(g, s));
+    }
+    for (int i = 0; i < count; ++i) {
+        const logq_status st = logq_linear(items[i].codes, items[i].cb, X, x_dtype, B, items[i].N, K, items[i].Y,
+                                           y_dtype, workspace, workspace_bytes, stream);
+        if (st != LOGQ_OK) return st;
+    }
+    return LOGQ_OK;
+}
+
 logq_status logq_workspace_status(void* workspace, void* stream, uint32_t* detail)
 {
     if (!workspace || !aligned16(workspace)) return LOGQ_ERR_WORKSPACE;

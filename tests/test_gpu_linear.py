@@ -159,3 +159,41 @@ def test_prefill_workspace_status_clean(logq):
     logq.logq_linear(codes, cb, X, N, K, workspace=ws)
     st, detail = logq.logq_workspace_status(ws)
     assert st == logq.LOGQ_OK and detail == 0
+
+
+@pytest.mark.parametrize("B", [1, 4, 16, 256])
+def test_grouped_matches_oracle(logq, B):
+    """q/k/v-like group sharing X (each matrix its own codebook), with an L2 warm-up range."""
+    K = 2048
+    shapes = [(2048, 1.35), (512, 1.8), (512, 1.5)]
+    layers = [make_layer(logq, N, K, 4, base, seed=70 + i) for i, (N, base) in enumerate(shapes)]
+    X = workloads.activations_torch(B, K, 77, torch.bfloat16, "cuda")
+    warm = torch.empty(3 << 20, dtype=torch.uint8, device="cuda")
+    items = [(codes, cb, N, None) for (codes, cb, ocb, q), (N, _) in zip(layers, shapes)]
+    outs = logq.logq_linear_grouped(items, X, K, prefetch=warm, prefetch_bytes=warm.numel())
+    for (codes, cb, ocb, q), Y in zip(layers, outs):
+        Yr, A = reference(X, q, ocb)
+        check_linear(Y.double().cpu().numpy(), Yr, A)
+
+
+@pytest.mark.parametrize("bits,B", [(3, 1), (3, 4), (4, 2)])
+def test_grouped_two_items_equal_single_calls(logq, bits, B):
+    K = 1152
+    a = make_layer(logq, 700, K, bits, 1.3, seed=81)
+    b = make_layer(logq, 300, K, bits, 1.7, seed=82)
+    X = workloads.activations_torch(B, K, 83, torch.bfloat16, "cuda")
+    ya, yb = logq.logq_linear_grouped([(a[0], a[1], 700, None), (b[0], b[1], 300, None)], X, K)
+    assert torch.equal(ya, logq.logq_linear(a[0], a[1], X, 700, K))
+    assert torch.equal(yb, logq.logq_linear(b[0], b[1], X, 300, K))
+
+
+def test_grouped_rejects_bad_groups(logq):
+    K = 256
+    a = make_layer(logq, 64, K, 4, 1.5, seed=90)
+    c = make_layer(logq, 64, K, 3, 1.5, seed=91)
+    X = workloads.activations_torch(1, K, 92, torch.bfloat16, "cuda")
+    with pytest.raises(logq.LogqError) as ei:
+        logq.logq_linear_grouped([(a[0], a[1], 64, None), (c[0], c[1], 64, None)], X, K)
+    assert ei.value.status == logq.LOGQ_ERR_INVALID_ARG
+    with pytest.raises(logq.LogqError):
+        logq.logq_linear_grouped([(a[0], a[1], 64, None)] * 5, X, K)
