@@ -471,8 +471,50 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+CASES = ("gemv_gateup_1b", "gemv_gate_8b", "prefill_q_8b", "quantize_gate_8b")
+
+
+def run_case(name: str):
+    """One small workload run twice (for a profiler capture of the second run):
+    the gate+up launch of the 1B decode step, the 8B gate GEMV, the 8B q-shaped
+    prefill GEMM (2048 tokens) and the quantisation of an 8B gate matrix."""
+    import torch
+    import paper_2607_01127_gb300 as logq
+    dev = torch.device("cuda", 0)
+    ws = logq.new_workspace(dev)
+    if name == "gemv_gateup_1b":
+        K = 2048
+        a = logq.logq_quantize(workloads.weights_torch(8192, K, 11, True, dev), 4, 1.4, workspace=ws)
+        b = logq.logq_quantize(workloads.weights_torch(8192, K, 12, True, dev), 4, 1.6, workspace=ws)
+        X = workloads.activations_torch(1, K, 1, torch.bfloat16, dev)
+        for _ in range(2):
+            logq.logq_linear_grouped([(a[0], a[1], 8192, None), (b[0], b[1], 8192, None)], X, K, workspace=ws)
+    elif name == "gemv_gate_8b":
+        N, K = workloads.LLAMA_8B_SHAPES["gate"]
+        c = logq.logq_quantize(workloads.weights_torch(N, K, 13, True, dev), 4, 1.5, workspace=ws)
+        X = workloads.activations_torch(1, K, 1, torch.bfloat16, dev)
+        for _ in range(2):
+            logq.logq_linear(c[0], c[1], X, N, K, workspace=ws)
+    elif name == "prefill_q_8b":
+        N, K = workloads.LLAMA_8B_SHAPES["q"]
+        c = logq.logq_quantize(workloads.weights_torch(N, K, 14, True, dev), 4, 1.5, workspace=ws)
+        X = workloads.activations_torch(PREFILL_TOKENS, K, 2, torch.bfloat16, dev)
+        for _ in range(2):
+            logq.logq_linear(c[0], c[1], X, N, K, y_dtype=torch.bfloat16, workspace=ws)
+    elif name == "quantize_gate_8b":
+        N, K = workloads.LLAMA_8B_SHAPES["gate"]
+        W = workloads.weights_torch(N, K, 15, True, dev)
+        for _ in range(2):
+            logq.logq_quantize(W, 4, 1.5, workspace=ws)
+    torch.cuda.synchronize()
+    st, _ = logq.logq_workspace_status(ws)
+    assert st == logq.LOGQ_OK
+    print("case", name, "ok")
+
+
 def main():
     ap = argparse.ArgumentParser()
+    ap.add_argument("--case", choices=CASES, help="run one small profiling case and exit")
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=10)
@@ -481,7 +523,9 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
-    if args.impl == "reference":
+    if args.case:
+        run_case(args.case)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_ours(args)

@@ -166,11 +166,6 @@ __device__ __forceinline__ void cp_async_4(uint32_t dst, const void* src)
     asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(dst), "l"(src) : "memory");
 }
 
-__device__ __forceinline__ void cp_async_8(uint32_t dst, const void* src)
-{
-    asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(dst), "l"(src) : "memory");
-}
-
 __device__ __forceinline__ void cp_async_16(uint32_t dst, const void* src)
 {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
@@ -249,13 +244,6 @@ __device__ __forceinline__ void sts128(uint32_t addr, uint32_t a, uint32_t b, ui
 {
     asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d)
                  : "memory");
-}
-
-__device__ __forceinline__ void store_y(void* Y, int dtype, int64_t idx, float v)
-{
-    if (dtype == LOGQ_F32) static_cast<float*>(Y)[idx] = v;
-    else if (dtype == LOGQ_BF16) static_cast<__nv_bfloat16*>(Y)[idx] = __float2bfloat16_rn(v);
-    else static_cast<__half*>(Y)[idx] = __float2half_rn(v);
 }
 
 // ------------------------------------------------------------------ kernel ---
@@ -446,10 +434,36 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
                 uint32_t v[32];
                 tmem_ld32(tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * kBN + c * 32), v);
                 if (n < p.N) {
+                    // lanes hold consecutive n: each store instruction writes one
+                    // contiguous run of Y[t][n0 .. n0+31]
+                    const int tb = t0 + c * 32;
+                    const int jmax = (p.B - tb) < 32 ? (p.B - tb) : 32;
+                    const int64_t base = (int64_t)tb * p.N + n;
+                    if (p.y_dtype == LOGQ_F32) {
+                        float* y = static_cast<float*>(p.Y) + base;
+                        if (jmax == 32) {
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        const int t = t0 + c * 32 + j;
-                        if (t < p.B) store_y(p.Y, p.y_dtype, (int64_t)t * p.N + n, __uint_as_float(v[j]));
+                            for (int j = 0; j < 32; ++j) y[(int64_t)j * p.N] = __uint_as_float(v[j]);
+                        } else {
+#pragma unroll
+                            for (int j = 0; j < 32; ++j)
+                                if (j < jmax) y[(int64_t)j * p.N] = __uint_as_float(v[j]);
+                        }
+                    } else if (p.y_dtype == LOGQ_BF16) {
+                        __nv_bfloat16* y = static_cast<__nv_bfloat16*>(p.Y) + base;
+                        if (jmax == 32) {
+#pragma unroll
+                            for (int j = 0; j < 32; ++j) y[(int64_t)j * p.N] = __float2bfloat16_rn(__uint_as_float(v[j]));
+                        } else {
+#pragma unroll
+                            for (int j = 0; j < 32; ++j)
+                                if (j < jmax) y[(int64_t)j * p.N] = __float2bfloat16_rn(__uint_as_float(v[j]));
+                        }
+                    } else {
+                        __half* y = static_cast<__half*>(p.Y) + base;
+#pragma unroll
+                        for (int j = 0; j < 32; ++j)
+                            if (j < jmax) y[(int64_t)j * p.N] = __float2half_rn(__uint_as_float(v[j]));
                     }
                 }
             }

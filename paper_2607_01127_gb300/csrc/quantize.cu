@@ -74,27 +74,32 @@ __global__ void __launch_bounds__(256) absmax_kernel(const float4* __restrict__ 
 }
 
 // Magnitude index of one weight: the number of boundaries not above |w|.
+// Boundaries are positive fp32 values, so they compare like their bit
+// patterns; |w| is compared as bits too (a NaN counts as large and is
+// reported separately).  q_max = 7 uses a three-step binary search, q_max = 3
+// a two-step one.
 template <int QMAX>
-__device__ __forceinline__ uint32_t magnitude(float w, const float (&t)[8])
+__device__ __forceinline__ uint32_t magnitude(uint32_t u, const uint32_t (&t)[8])
 {
-    const float a = fabsf(w);
-    uint32_t m = 0;
-#pragma unroll
-    for (int j = 0; j < QMAX; ++j) m += (a >= t[j]) ? 1u : 0u;
-    return m;
+    if constexpr (QMAX == 7) {
+        const bool b2 = u >= t[3];
+        const uint32_t t1 = b2 ? t[5] : t[1];
+        const bool b1 = u >= t1;
+        const uint32_t t0 = b2 ? (b1 ? t[6] : t[4]) : (b1 ? t[2] : t[0]);
+        return (b2 ? 4u : 0u) + (b1 ? 2u : 0u) + (u >= t0 ? 1u : 0u);
+    } else {
+        const bool b1 = u >= t[1];
+        const uint32_t t0 = b1 ? t[2] : t[0];
+        return (b1 ? 2u : 0u) + (u >= t0 ? 1u : 0u);
+    }
 }
 
 template <int BITS>
-__device__ __forceinline__ uint32_t code_of(float w, uint32_t m)
+__device__ __forceinline__ uint32_t code_of(uint32_t bits, uint32_t m)
 {
     // sign bit only for negative weights that did not round to zero
-    const uint32_t neg = (__float_as_uint(w) >> 31) & (m != 0 ? 1u : 0u);
-    return (neg << (BITS - 1)) | m;
-}
-
-__device__ __forceinline__ uint32_t nonfinite_of(float w)
-{
-    return (__float_as_uint(w) & 0x7f800000u) == 0x7f800000u ? 1u : 0u;
+    const uint32_t sign = (bits >> (32 - BITS)) & (1u << (BITS - 1));
+    return m != 0 ? (m | sign) : 0u;
 }
 
 // 4-bit: each thread turns 8 consecutive weights into one 32-bit word
@@ -103,10 +108,10 @@ __global__ void __launch_bounds__(256) quantize4_kernel(const float4* __restrict
                                                         QuantParams p, uint32_t* __restrict__ out,
                                                         Workspace* ws)
 {
-    float t[8];
+    uint32_t t[8];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) t[j] = p.thresh[j];
-    uint32_t bad = 0;
+    for (int j = 0; j < 8; ++j) t[j] = __float_as_uint(p.thresh[j]);
+    uint32_t umax = 0;                       // largest |w| bit pattern seen (non-finite check)
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nwords; i += stride) {
         const float4 a = ld_stream(W + 2 * i);
@@ -115,14 +120,15 @@ __global__ void __launch_bounds__(256) quantize4_kernel(const float4* __restrict
         uint32_t word = 0;
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
-            const uint32_t m = magnitude<7>(v[e], t);
-            word |= code_of<4>(v[e], m) << (4 * e);
-            bad |= nonfinite_of(v[e]);
+            const uint32_t bits = __float_as_uint(v[e]);
+            const uint32_t u = bits & 0x7fffffffu;
+            umax = max(umax, u);
+            word += code_of<4>(bits, magnitude<7>(u, t)) << (4 * e);   // disjoint nibbles: add = or
         }
         out[i] = word;
     }
     if (p.check_nonfinite) {
-        bad = __reduce_or_sync(0xffffffffu, bad);
+        const uint32_t bad = __reduce_or_sync(0xffffffffu, umax >= 0x7f800000u ? 1u : 0u);
         if (bad && (threadIdx.x & 31) == 0) atomicOr(&ws->nonfinite, 1u);
     }
 }
@@ -132,10 +138,10 @@ __global__ void __launch_bounds__(256) quantize3_kernel(const float4* __restrict
                                                         QuantParams p, uint32_t* __restrict__ out,
                                                         Workspace* ws)
 {
-    float t[8];
+    uint32_t t[8];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) t[j] = p.thresh[j];
-    uint32_t bad = 0;
+    for (int j = 0; j < 8; ++j) t[j] = __float_as_uint(p.thresh[j]);
+    uint32_t umax = 0;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < ngroups; g += stride) {
         uint32_t w0 = 0, w1 = 0, w2 = 0;
@@ -146,8 +152,10 @@ __global__ void __launch_bounds__(256) quantize3_kernel(const float4* __restrict
             uint32_t c[4];
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
-                c[e] = code_of<3>(v[e], magnitude<3>(v[e], t));
-                bad |= nonfinite_of(v[e]);
+                const uint32_t bits = __float_as_uint(v[e]);
+                const uint32_t u = bits & 0x7fffffffu;
+                umax = max(umax, u);
+                c[e] = code_of<3>(bits, magnitude<3>(u, t));
             }
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
@@ -170,7 +178,7 @@ __global__ void __launch_bounds__(256) quantize3_kernel(const float4* __restrict
         out[3 * g + 2] = w2;
     }
     if (p.check_nonfinite) {
-        bad = __reduce_or_sync(0xffffffffu, bad);
+        const uint32_t bad = __reduce_or_sync(0xffffffffu, umax >= 0x7f800000u ? 1u : 0u);
         if (bad && (threadIdx.x & 31) == 0) atomicOr(&ws->nonfinite, 1u);
     }
 }
