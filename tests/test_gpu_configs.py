@@ -1,0 +1,194 @@
+"""The five workloads at full size, checked against the fp64 oracle.
+
+  - Llama-3.2-1B decode step: all 16 layers' linears at batch 1 through the same
+    grouped launches the benchmark times, every output checked; codes bit-exact on
+    every layer.
+  - Llama-3.1-8B linears at batch 1, 4 and 16: every output checked.
+  - Llama-3.1-8B prefill (2048 tokens): sampled outputs computed one by one.
+  - Full 32-layer Llama-3.1-8B stack at 3 and 4 bits over bases 1.25, 1.5, 2.0:
+    every code checked against the oracle's fp64 decision boundaries (a property
+    that holds at any size), sampled rows bit-exact against the oracle's
+    quantiser, and a batch-1 pass through every linear checked on sampled rows.
+(The single 512 x 2048 layer is in test_gpu_quantize / test_gpu_linear.)
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2607_01127_gb300 import workloads
+
+from gpu_common import boundary_mask, check_linear, lib
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def logq():
+    return lib()
+
+
+def unpack_gpu(codes, N, K, bits):
+    """Signed integer codes [N, K] decoded from packed bytes with plain torch ops."""
+    c = codes.view(N, -1).to(torch.int32)
+    if bits == 4:
+        lo, hi = c & 15, c >> 4
+        nib = torch.stack([lo, hi], dim=2).reshape(N, K)
+        m, s = nib & 7, (nib >> 3) & 1
+    else:
+        g = c.view(N, K // 32, 12)
+        w = [g[..., 4 * i] | (g[..., 4 * i + 1] << 8) | (g[..., 4 * i + 2] << 16) | (g[..., 4 * i + 3] << 24)
+             for i in range(3)]
+        fields = []
+        for p in range(16):
+            if p < 15:
+                f = (w[p // 5] >> (6 * (p % 5))) & 63
+            else:
+                f = ((w[0] >> 30) & 3) | (((w[1] >> 30) & 3) << 2) | (((w[2] >> 30) & 3) << 4)
+            fields += [f & 7, f >> 3]
+        nib = torch.stack(fields, dim=2).reshape(N, K)
+        m, s = nib & 3, (nib >> 2) & 1
+    return torch.where(s == 1, -m, m)
+
+
+def check_codes_property(W, codes, ocb, bits):
+    """Every code's magnitude m must satisfy tau_{m-1} <= |w| < tau_m for the
+    oracle's fp64 boundaries (searchsorted, a library routine), and its sign must be
+    the weight's; mismatches are allowed only within one fp32 ulp of a boundary."""
+    N, K = W.shape
+    q = unpack_gpu(codes, N, K, bits)
+    taus = torch.tensor(ocb.taus, dtype=torch.float64, device=W.device)
+    a = W.abs().double()
+    m_ref = torch.searchsorted(taus, a, right=True)
+    q_ref = torch.where(W < 0, -m_ref, m_ref).to(torch.int32)
+    bad = q != q_ref
+    n_bad = int(bad.sum())
+    if n_bad:
+        wb = W[bad].cpu().numpy()
+        assert np.all(boundary_mask(wb, ocb)), "code mismatch away from a decision boundary"
+    return n_bad
+
+
+def check_rows_bit_exact(W, codes, ocb, bits, N, K, seed, count=4):
+    """Sampled rows: packed bytes equal the oracle's (log route) bit for bit, except
+    weights within one fp32 ulp of a boundary."""
+    rows = torch.from_numpy(sample_rows(N, count, seed)).cuda()
+    w_rows = W[rows].cpu().numpy()
+    got = codes.view(N, -1)[rows].cpu().numpy()
+    qw = oracle.quantize_log(w_rows, ocb)
+    if not np.array_equal(got, oracle.pack(qw, bits)):
+        qg = oracle.unpack(got, len(w_rows), K, bits)
+        assert np.all(boundary_mask(w_rows[qg != qw], ocb))
+    return rows
+
+
+def sample_rows(N, count, seed):
+    rng = np.random.Generator(np.random.PCG64(seed))
+    return np.unique(np.concatenate([[0, N - 1], rng.choice(N, size=min(count, N), replace=False)]))
+
+
+def test_config_llama1b_decode_step(logq):
+    """All 112 linears of the 1B-shaped decode step (grouped launches as in the
+    benchmark, each warming L2 with the next), every output checked."""
+    bases = workloads.layer_bases(workloads.LLAMA_1B_LAYERS, 1)
+    ws = logq.new_workspace()
+    for layer in range(workloads.LLAMA_1B_LAYERS):
+        lin = {}
+        for pi, name in enumerate(workloads.PROJ_NAMES):
+            N, K = workloads.LLAMA_1B_SHAPES[name]
+            W = workloads.weights_torch(N, K, workloads.layer_seed(1, layer, pi), outliers=True, device="cuda")
+            codes, cb = logq.logq_quantize(W, 4, float(bases[layer]), workspace=ws)
+            ocb = oracle.build_codebook(4, float(bases[layer]), float(W.abs().max()))
+            assert cb.range == ocb.range
+            assert check_codes_property(W, codes, ocb, 4) <= 4
+            check_rows_bit_exact(W, codes, ocb, 4, N, K, layer * 10 + pi)
+            lin[name] = (codes, cb, ocb, N, K)
+            del W
+        for grp in (("q", "k", "v"), ("o",), ("gate", "up"), ("down",)):
+            K = lin[grp[0]][4]
+            X = workloads.activations_torch(1, K, layer * 10 + len(grp), torch.bfloat16, "cuda")
+            outs = logq.logq_linear_grouped([(lin[n][0], lin[n][1], lin[n][3], None) for n in grp], X, K,
+                                            workspace=ws)
+            xd = X.float().cpu().double().numpy()
+            for n, Y in zip(grp, outs):
+                codes, cb, ocb, N, K = lin[n]
+                q = oracle.unpack(codes.cpu().numpy().reshape(N, -1), N, K, 4)
+                Yr, A = oracle.linear(xd, oracle.dequant(q, ocb, oracle.TABLE_BF16))
+                check_linear(Y.double().cpu().numpy(), Yr, A)
+    st, _ = logq.logq_workspace_status(ws)
+    assert st == logq.LOGQ_OK
+
+
+@pytest.mark.parametrize("B", [1, 4, 16])
+def test_config_llama8b_decode_batches(logq, B):
+    ws = logq.new_workspace()
+    for pi, name in enumerate(workloads.PROJ_NAMES):
+        if name in ("v", "up"):
+            continue                         # same shapes as k and gate
+        N, K = workloads.LLAMA_8B_SHAPES[name]
+        W = workloads.weights_torch(N, K, workloads.layer_seed(3, 0, pi), outliers=False, device="cuda")
+        base = 1.2 + 0.1 * pi
+        codes, cb = logq.logq_quantize(W, 4, base, workspace=ws)
+        ocb = oracle.build_codebook(4, base, float(W.abs().max()))
+        assert check_codes_property(W, codes, ocb, 4) <= 4
+        del W
+        X = workloads.activations_torch(B, K, pi, torch.bfloat16, "cuda")
+        Y = logq.logq_linear(codes, cb, X, N, K, workspace=ws)
+        q = oracle.unpack(codes.cpu().numpy().reshape(N, -1), N, K, 4)
+        Yr, A = oracle.linear(X.float().cpu().double().numpy(), oracle.dequant(q, ocb, oracle.TABLE_BF16))
+        check_linear(Y.double().cpu().numpy(), Yr, A)
+
+
+def test_config_llama8b_prefill(logq):
+    """2048 tokens through each 8B linear shape (the benchmark's prefill leg),
+    sampled outputs computed one by one by the oracle."""
+    T = 2048
+    ws = logq.new_workspace()
+    rng = np.random.Generator(np.random.PCG64(44))
+    for pi, name in enumerate(workloads.PROJ_NAMES):
+        if name in ("v", "up"):
+            continue
+        N, K = workloads.LLAMA_8B_SHAPES[name]
+        W = workloads.weights_torch(N, K, workloads.layer_seed(4, 0, pi), outliers=True, device="cuda")
+        codes, cb = logq.logq_quantize(W, 4, 1.5, workspace=ws)
+        del W
+        ocb = oracle.build_codebook(4, 1.5, cb.range)
+        X = workloads.activations_torch(T, K, pi, torch.bfloat16, "cuda")
+        Y = logq.logq_linear(codes, cb, X, N, K, y_dtype=torch.bfloat16, workspace=ws)
+        bs = np.concatenate([rng.integers(0, T, 3000), np.zeros(64, np.int64), np.full(64, T - 1)])
+        ns = np.concatenate([rng.integers(0, N, 3000), rng.integers(0, N, 128)])
+        Yr, A = oracle.linear_sampled(X.float().cpu().double().numpy(), codes.cpu().numpy(), 4, ocb,
+                                      oracle.TABLE_BF16, bs, ns, nthreads=0)
+        got = Y.float().cpu().double().numpy()[bs, ns]
+        check_linear(got[None], Yr[None], A[None], "bf16")
+    st, _ = logq.logq_workspace_status(ws)
+    assert st == logq.LOGQ_OK
+
+
+@pytest.mark.parametrize("bits", [3, 4])
+@pytest.mark.parametrize("base", [1.25, 1.5, 2.0])
+def test_config_llama8b_full_stack(logq, bits, base):
+    """All 224 linears of the 32-layer 8B-shaped stack quantised at (bits, base),
+    then a batch-1 pass through every linear, checked layer by layer."""
+    ws = logq.new_workspace()
+    n_boundary = 0
+    for layer in range(workloads.LLAMA_8B_LAYERS):
+        for pi, name in enumerate(workloads.PROJ_NAMES):
+            N, K = workloads.LLAMA_8B_SHAPES[name]
+            seed = workloads.layer_seed(5, layer, pi)
+            W = workloads.weights_torch(N, K, seed, outliers=True, device="cuda")
+            codes, cb = logq.logq_quantize(W, bits, base, workspace=ws)
+            ocb = oracle.build_codebook(bits, base, float(W.abs().max()))
+            assert cb.range == ocb.range
+            if (bits == 4 and base == 1.5) or layer % 8 == 0:     # every element, every 8th layer otherwise
+                n_boundary += check_codes_property(W, codes, ocb, bits)
+            rows = check_rows_bit_exact(W, codes, ocb, bits, N, K, seed, count=6)
+            del W
+            X = workloads.activations_torch(1, K, seed, torch.bfloat16, "cuda")
+            Y = logq.logq_linear(codes, cb, X, N, K, workspace=ws)
+            sub = codes.view(N, -1)[rows].cpu().numpy()
+            ns = np.arange(len(sub), dtype=np.int64)
+            Yr, A = oracle.linear_sampled(X.float().cpu().double().numpy(), sub, bits, ocb,
+                                          oracle.TABLE_BF16, np.zeros_like(ns), ns)
+            check_linear(Y[0, rows].double().cpu().numpy()[None], Yr[None], A[None])
+    assert n_boundary <= 32
