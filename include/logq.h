@@ -28,6 +28,12 @@
  *   - Every argument is validated before anything is enqueued.  A call that
  *     returns an error other than LOGQ_ERR_CUDA / LOGQ_ERR_NONFINITE has
  *     touched no device memory.
+ *   - Decode launches (logq_linear with small B, logq_linear_grouped) use
+ *     programmatic dependent launch: they may start while the preceding kernel
+ *     on the stream finishes.  They read X and write Y only after that kernel
+ *     has completed, but may read the packed codes earlier; codes written by
+ *     a kernel that signals early completion (griddepcontrol.launch_dependents)
+ *     must be ordered before the call by other means (e.g. an event or a copy).
  *   - Device code never traps.  Conditions found on the device (non-finite
  *     weights, a pipeline wait that exceeded its bound) are written to the
  *     caller's workspace and reported by logq_quantize or logq_workspace_status.

@@ -70,6 +70,7 @@ struct GemvParams {
     int32_t chunk_rows;   // rows reduced per shared-memory pass
     const uint8_t* pf;    // optional L2 warm-up range (e.g. the next layer's codes)
     int64_t pf_bytes;
+    int64_t pf_share;     // bytes of that range per CTA (multiple of 16)
 };
 
 __device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel)
@@ -268,6 +269,40 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
     const int64_t r0 = (int64_t)c * item.rows_q + (c < item.rows_rem ? c : item.rows_rem);
     const int64_t r1 = r0 + item.rows_q + (c < item.rows_rem ? 1 : 0);
 
+    // 0) the first round of code loads of this warp's first (chunk, span) goes
+    //    out first: its latency hides behind the prologue below.  Codes are
+    //    weights, not the previous kernel's output (see the launch contract).
+    const int G = p.groups, SC = p.span_cols;
+    const bool compute_warp = warp < G * SC;
+    const int g = warp % G, scol = warp / G;
+    const int64_t rstride = (int64_t)G * p.row_bytes;
+    CodeVec<NW> ca[R], cb[R];
+    auto span_first = [&](int64_t q0, int s, int& k0, bool& active) -> const uint8_t* {
+        k0 = s * SPAN + lane * KW;
+        active = k0 < p.K;
+        // idle lanes read the row start (valid memory) and multiply by zero
+        const int64_t lane_byte = active ? ((BITS == 4) ? (int64_t)k0 / 2 : (int64_t)k0 / 32 * 12) : 0;
+        return item.codes + (q0 + g) * p.row_bytes + lane_byte;
+    };
+    auto load_round = [&](CodeVec<NW> (&c)[R], const uint8_t* first, int my_rows, int t) {
+        const int here = my_rows - t * R;
+        const uint8_t* rp = first + (int64_t)t * R * rstride;
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+            if (r < here) c[r] = ld_codes<NW>(rp + (int64_t)r * rstride);
+    };
+    bool preloaded = false;                     // ca holds the first round of the first (chunk, span)
+    {
+        const int nrows0 = (int)((r0 + p.chunk_rows < r1 ? r0 + p.chunk_rows : r1) - r0);
+        const int my_rows0 = (nrows0 > g) ? (nrows0 - g + G - 1) / G : 0;
+        if (compute_warp && my_rows0 > 0 && scol < p.spans) {
+            int k0;
+            bool active;
+            load_round(ca, span_first(r0, scol, k0, active), my_rows0, 0);
+            preloaded = true;
+        }
+    }
+
     // 1) start streaming this CTA's code rows into L2, and its share of the
     //    optional warm-up range.
     {
@@ -281,9 +316,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                          : "memory");
         }
         if (p.pf_bytes > 0) {
-            const int64_t share = ((p.pf_bytes + gridDim.x - 1) / gridDim.x + 15) & ~(int64_t)15;
-            const int64_t beg = share * blockIdx.x;
-            const int64_t end = (beg + share < p.pf_bytes) ? beg + share : p.pf_bytes;
+            const int64_t beg = p.pf_share * blockIdx.x;
+            const int64_t end = (beg + p.pf_share < p.pf_bytes) ? beg + p.pf_share : p.pf_bytes;
             for (int64_t off = beg + (int64_t)tid * piece; off < end; off += (int64_t)kThreads * piece) {
                 const int64_t n = (end - off) < piece ? (end - off) : piece;
                 asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p.pf + off), "r"((uint32_t)n)
@@ -301,30 +335,31 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
     float* red = (tab_addr - sbase >= red_bytes) ? reinterpret_cast<float*>(smem)
                                                  : reinterpret_cast<float*>(smem + (tab_addr - sbase) + TAB_BYTES);
     // entry e = (value of its low code) | (value of its high code) << 16,
-    // 32 copies (one per lane) in the first 128 bytes of its 256-byte row.
+    // 32 copies (one per lane) in the first 128 bytes of its 256-byte row.  The
+    // 16 levels are staged in shared memory first (indexed parameter reads
+    // with per-thread indices would serialise).
+    __shared__ uint32_t s_lvl[16];
+    if (tid < 16) s_lvl[tid] = item.lvl16[tid] & 0xffffu;
+    __syncthreads();
     for (int i = tid; i < NENT * 8; i += kThreads) {
         const int e = i >> 3, part = i & 7;
         const uint32_t lo = (BITS == 4) ? (e & 15) : (e & 7);
         const uint32_t hi = (BITS == 4) ? (e >> 4) : (e >> 3);
-        const uint32_t v = (item.lvl16[lo] & 0xffffu) | (item.lvl16[hi] << 16);
+        const uint32_t v = s_lvl[lo] | (s_lvl[hi] << 16);
         reinterpret_cast<uint4*>(tab + e * (kTabStride / 4))[part] = make_uint4(v, v, v, v);
     }
     __syncthreads();
-    // 3) programmatic dependent launch: everything above touched only kernel
-    //    parameters, shared memory and an L2 hint, so it may overlap the tail of
-    //    the previous kernel on the stream.  X may be that kernel's output and Y
-    //    its input: wait for it before the first global read or write.
+    // 3) programmatic dependent launch: the work above and the first code
+    //    loads below touch only parameters, shared memory and the weights, so
+    //    they may overlap the tail of the previous kernel on the stream.  X may be
+    //    that kernel's output and Y its input: every thread waits for it before
+    //    its first read of X or write of Y.
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-    asm volatile("griddepcontrol.wait;" ::: "memory");
 
     const uint32_t base_lane = tab_addr | (4u * (uint32_t)lane);
-    const int G = p.groups, SC = p.span_cols;
-    const bool compute_warp = warp < G * SC;
-    const int g = warp % G, scol = warp / G;
     constexpr int lg2V = (V >= 32) ? 5 : (V >= 16) ? 4 : (V >= 8) ? 3 : (V >= 4) ? 2 : (V >= 2) ? 1 : 0;
     const int my_v = lane >> (5 - lg2V);
     const bool writer = (lane & ((32 >> lg2V) - 1)) == 0;
-    const int64_t rstride = (int64_t)G * p.row_bytes;
 
     for (int64_t q0 = r0; q0 < r1; q0 += p.chunk_rows) {
         const int64_t q1 = (q0 + p.chunk_rows < r1) ? q0 + p.chunk_rows : r1;
@@ -333,8 +368,15 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
         const int nrounds = (my_rows + R - 1) / R;
         if (compute_warp && my_rows > 0) {
             for (int s = scol; s < p.spans; s += SC) {
-                const int k0 = s * SPAN + lane * KW;
-                const bool active = k0 < p.K;
+                int k0;
+                bool active;
+                const uint8_t* first = span_first(q0, s, k0, active);
+                // Rounds of R rows with two code buffers: the loads of round t+1 are
+                // in flight while round t is decoded.  Full rounds run unguarded;
+                // the last round guards its rows (warp-uniform branches).
+                if (!preloaded) load_round(ca, first, my_rows, 0);
+                preloaded = false;
+                asm volatile("griddepcontrol.wait;" ::: "memory");
                 // activations for this span stay in registers (zero on idle lanes)
                 uint32_t xr[B][NPAIR];
 #pragma unroll
@@ -350,21 +392,6 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                         if (i + 3 < NPAIR) xr[b][i + 3] = v.w;
                     }
                 }
-                // idle lanes read the row start (valid memory) and multiply by zero
-                const int64_t lane_byte = active ? ((BITS == 4) ? (int64_t)k0 / 2 : (int64_t)k0 / 32 * 12) : 0;
-                const uint8_t* first = item.codes + (q0 + g) * p.row_bytes + lane_byte;
-
-                // Rounds of R rows with two code buffers: the loads of round t+1 are
-                // in flight while round t is decoded.  Full rounds run unguarded;
-                // the last round guards its rows (warp-uniform branches).
-                CodeVec<NW> ca[R], cb[R];
-                auto load_round = [&](CodeVec<NW> (&c)[R], int t) {
-                    const int here = my_rows - t * R;
-                    const uint8_t* rp = first + (int64_t)t * R * rstride;
-#pragma unroll
-                    for (int r = 0; r < R; ++r)
-                        if (r < here) c[r] = ld_codes<NW>(rp + (int64_t)r * rstride);
-                };
                 auto run_round = [&](const CodeVec<NW> (&c)[R], int t) {
                     const int here = my_rows - t * R;
                     float acc[V], acc_hi[V];
@@ -387,16 +414,16 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                         if (lr < nrows) red[((int64_t)s * p.chunk_rows + lr) * B + b] = acc[0];
                     }
                 };
-                load_round(ca, 0);
                 for (int t = 0; t < nrounds; t += 2) {
-                    if (t + 1 < nrounds) load_round(cb, t + 1);
+                    if (t + 1 < nrounds) load_round(cb, first, my_rows, t + 1);
                     run_round(ca, t);
                     if (t + 1 >= nrounds) break;
-                    if (t + 2 < nrounds) load_round(ca, t + 2);
+                    if (t + 2 < nrounds) load_round(ca, first, my_rows, t + 2);
                     run_round(cb, t + 1);
                 }
             }
         }
+        asm volatile("griddepcontrol.wait;" ::: "memory");
         __syncthreads();
         // fixed-order sum over spans
         for (int i = tid; i < nrows * B; i += kThreads) {
@@ -553,6 +580,7 @@ cudaError_t launch_gemv_group(const GroupArgs& a, cudaStream_t s)
         --used;
     }
     grid = used;
+    p.pf_share = p.pf_bytes > 0 ? (((p.pf_bytes + grid - 1) / grid + 15) & ~(int64_t)15) : 0;
     int64_t max_rows = 0;
     int begin = 0;
     for (int i = 0; i < a.count; ++i) {
