@@ -302,6 +302,20 @@ def time_prefill(logq, torch, dev, reps: int = 3):
     return {"layers": res, "tflops": tot_flop / tot_t / 1e12}
 
 
+def replica_totals(t_local: float, units_local: float, dist=None, device=None):
+    """Whole-job throughput of N independent replicas: every rank processed
+    units_local in t_local seconds; the job takes as long as the slowest rank.
+    Returns (max time over ranks, total units over ranks)."""
+    import torch
+    if dist is None or not dist.is_initialized() or dist.get_world_size() == 1:
+        return t_local, units_local
+    t = torch.tensor([t_local], dtype=torch.float64, device=device)
+    u = torch.tensor([units_local], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(u, op=dist.ReduceOp.SUM)
+    return float(t.item()), float(u.item())
+
+
 def run_ours(args):
     import torch
     import paper_2607_01127_gb300 as logq
@@ -357,12 +371,8 @@ def run_ours(args):
             e1.record(stream)
         barrier()
         time.sleep(0.25)
-    t = e0.elapsed_time(e1) * 1e-3
-    if dist is not None:
-        tt = torch.tensor([t], device=dev, dtype=torch.float64)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        t = float(tt.item())
-    value = step_bytes * args.steps * world / t / 1e9
+    t, total_bytes = replica_totals(e0.elapsed_time(e1) * 1e-3, step_bytes * args.steps, dist, dev)
+    value = total_bytes / t / 1e9
     ms_per_step = t / args.steps * 1e3
 
     # e2e: activations from pinned host memory in, outputs to host out, every step
@@ -405,12 +415,8 @@ def run_ours(args):
             yh.copy_(yd, non_blocking=True)
         f1.record(stream)
     barrier()
-    t2 = f0.elapsed_time(f1) * 1e-3
-    if dist is not None:
-        tt = torch.tensor([t2], device=dev, dtype=torch.float64)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        t2 = float(tt.item())
-    e2e_value = step_bytes * args.steps * world / t2 / 1e9
+    t2, total_bytes2 = replica_totals(f0.elapsed_time(f1) * 1e-3, step_bytes * args.steps, dist, dev)
+    e2e_value = total_bytes2 / t2 / 1e9
     # the e2e output equals the device-resident run
     first = launches[0]["members"][0]
     assert torch.equal(yd[:first["N"]], first["Y"].view(-1))
