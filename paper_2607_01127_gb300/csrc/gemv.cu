@@ -1,21 +1,28 @@
 // Decode GEMV / skinny GEMM on CUDA cores: Y[b][n] = sum_k X[b][k] * table[code(n, k)]
 // (paper Sec. 3.3: dequantisation by lookup table instead of exponentiation).
 //
-// Design (one persistent CTA of 16 warps per SM):
+// Design (CTAs of 8 or 16 warps, see the launch shapes below):
 //  * Pair table in shared memory.  Two codes (one byte at 4 bits, one 6-bit
 //    field at 3 bits) index a table whose entry is the bf16x2 / f16x2 pair of
 //    their dequantised values, signs included.  Each entry occupies a 256-byte
 //    row holding one copy per lane, so lane l always reads bank l: the lookups
-//    of a warp never conflict.  At 4 bits the byte offset of an entry,
-//    byte << 8 | 4 * lane, is one byte permute (prmt) of the code word.
+//    of a warp never conflict.  The table starts the dynamic shared memory at
+//    the fixed shared address kTabOff, so the byte offset of an entry,
+//    byte << 8 | 4 * lane, is one byte permute (prmt) of the code word and the
+//    table base is the load's immediate offset.
 //  * Each warp owns a fixed span of K (32 lanes x KW consecutive k) and keeps
 //    its activations for that span in registers for the whole kernel; it walks
 //    the rows of the CTA's row range, one 16-, 8- or 4-byte coalesced load of
 //    codes per lane and row (a warp reads a contiguous 512/256/128-byte run).
-//  * fp32 accumulation (mixed-precision fma with bf16/f16 operands, or packed
-//    fp32 fma after unpacking), a reduce-scatter across the 32 lanes per round
-//    of rows, then a fixed-order sum over the spans in shared memory: results
-//    are bit-identical from run to run.
+//  * fp32 accumulation (mixed-precision fma with bf16/f16 operands), a
+//    reduce-scatter across the 32 lanes per round of rows, then a fixed-order
+//    sum over the spans in shared memory: results are bit-identical from run
+//    to run.
+//  * Small launches run one 8-warp CTA per SM, which leaves room for the CTAs
+//    of the next launch on the stream: with programmatic dependent launch
+//    they start beside this one and build their table and issue their first
+//    code loads while it runs.  Large launches run one 16-warp CTA per SM to
+//    keep enough loads in flight; batches of 4 and more two 8-warp CTAs.
 //  * The CTA's contiguous range of code rows is prefetched into L2 with bulk
 //    prefetches at kernel start, so HBM streams at full rate while the warps
 //    consume from L2.
@@ -26,22 +33,42 @@
 
 #include "internal.h"
 
-#ifndef LOGQ_GEMV_FMA_MODE
-#define LOGQ_GEMV_FMA_MODE 0   // 0: fma.rn.f32.{bf16,f16}; 1: fma.rn.f32x2 on unpacked bf16
-#endif
-
 namespace logq {
 namespace {
 
-constexpr int kThreads = 512;
-constexpr int kWarps = kThreads / 32;
+// Threads per CTA: 256 (two CTAs fit on an SM) for small launches and
+// batches of 4 and more, 512 (one per SM, all 16 warps sharing one table) for
+// large batch-1/2 launches.
+constexpr int kSmallThreads = 256;
+constexpr int kLargeThreads = 512;
 constexpr int kTabStride = 256;               // bytes per pair-table entry
-constexpr int kRedBytes = 60 * 1024;          // span-partial buffer
+// Shared address at which dynamic shared memory starts in a kernel without
+// static shared memory: the per-CTA reserved area comes first.
+constexpr uint32_t kTabOff = 1024;
+constexpr uint32_t kLvlOff = 128;             // levels staged in the free half of table row 0
+// Span partials: for batch 1-2 at 4 bits they live in the free upper halves
+// of the table's 256 rows (32 KiB), otherwise after the table.
+constexpr int kRedBytes = 32 * 1024;
+__host__ __device__ constexpr bool red_in_table(int bits, int B) { return bits == 4 && B <= 2; }
 constexpr int64_t kPrefetchCap = 1 << 20;     // bytes of codes prefetched per CTA up front
-// table (64 KiB at 4 bits) + up to 64 KiB of alignment pad + span partials
-constexpr int kMaxSmem = 65536 + 256 * kTabStride + kRedBytes;
-
+constexpr int kMaxSmem = 256 * kTabStride + kRedBytes;
 constexpr int kMaxItems = 4;
+// Launches with at least this many bytes of codes run 16 warps per SM: their
+// main loop needs them to keep enough loads in flight.  Smaller launches run
+// 8 warps per SM, leaving the other half of the SM to the next launch.
+#ifndef LOGQ_GEMV_SPLIT_BYTES
+#define LOGQ_GEMV_SPLIT_BYTES (20 << 20)
+#endif
+constexpr int64_t kSplitBytes = LOGQ_GEMV_SPLIT_BYTES;
+// Shared-memory carveout of the batch-1/2 decode kernels, in percent of the
+// maximum: 58 % is 132 KiB, room for two CTAs of 64 KiB (plus their reserved
+// 1 KiB).  The rest of the 256 KiB per SM is L1, which also holds the data of
+// the code loads in flight, so a larger carveout slows the kernel down; one
+// setting for all of them spares the SMs a reconfiguration between launches.
+// Batches of 4 and more (two CTAs of up to 97 KiB) take the largest one.
+#ifndef LOGQ_GEMV_CARVEOUT
+#define LOGQ_GEMV_CARVEOUT 58
+#endif
 
 // One matrix of a grouped launch: all items share X, K, B and the code width.
 struct GemvItem {
@@ -63,6 +90,7 @@ struct GemvParams {
     int32_t B;
     int32_t y_dtype;
     const uint16_t* X;
+    uint32_t* err;        // workspace error word
     int64_t row_bytes;
     int32_t spans;        // S: spans of 32*KW k covering K
     int32_t groups;       // G: warps sharing one span (row-parallel)
@@ -80,10 +108,11 @@ __device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel)
     return r;
 }
 
-__device__ __forceinline__ uint32_t lds32(uint32_t addr)
+// Table entry at byte offset off from the table base.
+__device__ __forceinline__ uint32_t lds_tab(uint32_t off)
 {
     uint32_t v;
-    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr));
+    asm volatile("ld.shared.u32 %0, [%1+%2];" : "=r"(v) : "r"(off), "n"(kTabOff));
     return v;
 }
 
@@ -111,7 +140,6 @@ __device__ __forceinline__ CodeVec<NW> ld_codes(const uint8_t* p)
 template <bool F16>
 __device__ __forceinline__ void fma_pair(float& a0, float& a1, uint32_t w, uint32_t x)
 {
-#if LOGQ_GEMV_FMA_MODE == 0
     if constexpr (F16) {
         asm("{.reg .b16 wl, wh, xl, xh;\n\t"
             "mov.b32 {wl, wh}, %2;\n\t"
@@ -127,27 +155,6 @@ __device__ __forceinline__ void fma_pair(float& a0, float& a1, uint32_t w, uint3
             "fma.rn.f32.bf16 %1, wh, xh, %1;}"
             : "+f"(a0), "+f"(a1) : "r"(w), "r"(x));
     }
-#else
-    if constexpr (F16) {
-        asm("{.reg .b16 wl, wh, xl, xh;\n\t"
-            "mov.b32 {wl, wh}, %2;\n\t"
-            "mov.b32 {xl, xh}, %3;\n\t"
-            "fma.rn.f32.f16 %0, wl, xl, %0;\n\t"
-            "fma.rn.f32.f16 %1, wh, xh, %1;}"
-            : "+f"(a0), "+f"(a1) : "r"(w), "r"(x));
-    } else {
-        // bf16 -> fp32 is a 16-bit shift; x arrives unpacked the same way.
-        const float wl = __uint_as_float(w << 16), wh = __uint_as_float(w & 0xffff0000u);
-        const float xl = __uint_as_float(x << 16), xh = __uint_as_float(x & 0xffff0000u);
-        asm("{.reg .b64 a, b, c;\n\t"
-            "mov.b64 a, {%2, %3};\n\t"
-            "mov.b64 b, {%4, %5};\n\t"
-            "mov.b64 c, {%0, %1};\n\t"
-            "fma.rn.f32x2 c, a, b, c;\n\t"
-            "mov.b64 {%0, %1}, c;}"
-            : "+f"(a0), "+f"(a1) : "f"(wl), "f"(wh), "f"(xl), "f"(xh));
-    }
-#endif
 }
 
 // Reduce V per-lane values over the 32 lanes; afterwards lane l holds the
@@ -187,9 +194,9 @@ __device__ __forceinline__ void store_y(void* Y, int dtype, int64_t idx, float v
     }
 }
 
-// Shared-memory addresses of the four pair entries of one 4-bit code word.
-// base_lane holds 4 * lane in byte 0 and the table's 64 KiB-aligned shared
-// address in bytes 2-3, so one byte permute yields table + byte * 256 + 4 * lane.
+// Table offsets of the four pair entries of one 4-bit code word: base_lane
+// holds 4 * lane in byte 0 and zeros above, so one byte permute yields
+// byte * 256 + 4 * lane.
 __device__ __forceinline__ void addrs4(uint32_t c, uint32_t base_lane, uint32_t (&o)[4])
 {
     o[0] = prmt(c, base_lane, 0x7604u);
@@ -198,8 +205,8 @@ __device__ __forceinline__ void addrs4(uint32_t c, uint32_t base_lane, uint32_t 
     o[3] = prmt(c, base_lane, 0x7634u);
 }
 
-// Addresses of the 16 pair entries of one 3-bit group (W0, W1, W2); the
-// 6-bit field lands in bits 8-13, base_lane supplies the rest.
+// Table offsets of the 16 pair entries of one 3-bit group (W0, W1, W2); the
+// 6-bit field lands in bits 8-13, base_lane supplies 4 * lane.
 __device__ __forceinline__ void addrs3(const uint32_t (&w)[3], uint32_t base_lane, uint32_t (&o)[16])
 {
 #pragma unroll
@@ -225,7 +232,7 @@ __device__ __forceinline__ void decode_row(const CodeVec<NW>& c, uint32_t base_l
             addrs4(c.w[wi], base_lane, o);
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
-                const uint32_t wp = lds32(o[j]);
+                const uint32_t wp = lds_tab(o[j]);
 #pragma unroll
                 for (int b = 0; b < B; ++b) fma_pair<F16>(acc[b], acc_hi[b], wp, xr[b][4 * wi + j]);
             }
@@ -238,7 +245,7 @@ __device__ __forceinline__ void decode_row(const CodeVec<NW>& c, uint32_t base_l
             addrs3(w3, base_lane, o);
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
-                const uint32_t wp = lds32(o[j]);
+                const uint32_t wp = lds_tab(o[j]);
 #pragma unroll
                 for (int b = 0; b < B; ++b) fma_pair<F16>(acc[b], acc_hi[b], wp, xr[b][16 * gi + j]);
             }
@@ -246,8 +253,8 @@ __device__ __forceinline__ void decode_row(const CodeVec<NW>& c, uint32_t base_l
     }
 }
 
-template <int BITS, int B, int KW, int R, bool F16>
-__global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant__ GemvParams p)
+template <int BITS, int B, int KW, int R, bool F16, int NT>
+__global__ void __launch_bounds__(NT, 512 / NT) gemv_kernel(const __grid_constant__ GemvParams p)
 {
     extern __shared__ __align__(16) uint8_t smem[];
     constexpr int NPAIR = KW / 2;                            // bf16 pairs of x per lane and batch row
@@ -258,7 +265,16 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
     constexpr int SPAN = 32 * KW;
     static_assert(V <= 32 && (V & (V - 1)) == 0, "values per lane must be a power of two <= 32");
 
+    // programmatic dependent launch: the next kernel on the stream may start
+    // now.  Its CTAs may run beside this one and do their own prologue
+    // meanwhile; they wait for this grid to finish before they touch X or Y.
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    if ((uint32_t)__cvta_generic_to_shared(smem) != kTabOff) {   // table addressing relies on it
+        if (tid == 0) atomicExch(p.err, (uint32_t)LOGQ_ERR_UNSUPPORTED);
+        return;
+    }
     // this CTA's matrix and its contiguous range of rows
     int m = 0;
 #pragma unroll
@@ -310,7 +326,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
         const uint8_t* base = item.codes + r0 * p.row_bytes;
         int64_t bytes = (r1 - r0) * p.row_bytes;
         if (bytes > kPrefetchCap) bytes = kPrefetchCap;
-        for (int64_t off = (int64_t)tid * piece; off < bytes; off += (int64_t)kThreads * piece) {
+        for (int64_t off = (int64_t)tid * piece; off < bytes; off += (int64_t)NT * piece) {
             const int64_t n = (bytes - off) < piece ? (bytes - off) : piece;
             asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base + off), "r"((uint32_t)n)
                          : "memory");
@@ -318,7 +334,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
         if (p.pf_bytes > 0) {
             const int64_t beg = p.pf_share * blockIdx.x;
             const int64_t end = (beg + p.pf_share < p.pf_bytes) ? beg + p.pf_share : p.pf_bytes;
-            for (int64_t off = beg + (int64_t)tid * piece; off < end; off += (int64_t)kThreads * piece) {
+            for (int64_t off = beg + (int64_t)tid * piece; off < end; off += (int64_t)NT * piece) {
                 const int64_t n = (end - off) < piece ? (end - off) : piece;
                 asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p.pf + off), "r"((uint32_t)n)
                              : "memory");
@@ -326,37 +342,30 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
         }
     }
 
-    // 2) pair table at the first 64 KiB-aligned shared address of the
-    //    allocation; the span partials go below it when they fit, else above.
-    const uint32_t sbase = (uint32_t)__cvta_generic_to_shared(smem);
-    const uint32_t tab_addr = (sbase + 0xffffu) & ~0xffffu;
-    uint32_t* tab = reinterpret_cast<uint32_t*>(smem + (tab_addr - sbase));
-    const uint32_t red_bytes = (uint32_t)p.spans * (uint32_t)p.chunk_rows * B * 4u;
-    float* red = (tab_addr - sbase >= red_bytes) ? reinterpret_cast<float*>(smem)
-                                                 : reinterpret_cast<float*>(smem + (tab_addr - sbase) + TAB_BYTES);
-    // entry e = (value of its low code) | (value of its high code) << 16,
-    // 32 copies (one per lane) in the first 128 bytes of its 256-byte row.  The
-    // 16 levels are staged in shared memory first (indexed parameter reads
-    // with per-thread indices would serialise).
-    __shared__ uint32_t s_lvl[16];
-    if (tid < 16) s_lvl[tid] = item.lvl16[tid] & 0xffffu;
+    // 2) pair table: entry e = (value of its low code) | (value of its high
+    //    code) << 16, 32 copies (one per lane) in the first 128 bytes of its
+    //    256-byte row.  The 16 levels are staged in the free half of row 0
+    //    (indexed parameter reads with per-thread indices would serialise).
+    uint32_t* lvl = reinterpret_cast<uint32_t*>(smem + kLvlOff);
+    if (tid < 16) lvl[tid] = item.lvl16[tid] & 0xffffu;
     __syncthreads();
-    for (int i = tid; i < NENT * 8; i += kThreads) {
+    for (int i = tid; i < NENT * 8; i += NT) {
         const int e = i >> 3, part = i & 7;
         const uint32_t lo = (BITS == 4) ? (e & 15) : (e & 7);
         const uint32_t hi = (BITS == 4) ? (e >> 4) : (e >> 3);
-        const uint32_t v = s_lvl[lo] | (s_lvl[hi] << 16);
-        reinterpret_cast<uint4*>(tab + e * (kTabStride / 4))[part] = make_uint4(v, v, v, v);
+        const uint32_t v = lvl[lo] | (lvl[hi] << 16);
+        reinterpret_cast<uint4*>(smem + e * kTabStride)[part] = make_uint4(v, v, v, v);
     }
+    // span partial i (in the free half of table row i / 32, or after the table)
+    auto red = [&](int i) -> float& {
+        if constexpr (red_in_table(BITS, B))
+            return *reinterpret_cast<float*>(smem + (i >> 5) * kTabStride + 128 + (i & 31) * 4);
+        else
+            return reinterpret_cast<float*>(smem + TAB_BYTES)[i];
+    };
     __syncthreads();
-    // 3) programmatic dependent launch: the work above and the first code
-    //    loads below touch only parameters, shared memory and the weights, so
-    //    they may overlap the tail of the previous kernel on the stream.  X may be
-    //    that kernel's output and Y its input: every thread waits for it before
-    //    its first read of X or write of Y.
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
-    const uint32_t base_lane = tab_addr | (4u * (uint32_t)lane);
+    const uint32_t base_lane = 4u * (uint32_t)lane;
     constexpr int lg2V = (V >= 32) ? 5 : (V >= 16) ? 4 : (V >= 8) ? 3 : (V >= 4) ? 2 : (V >= 2) ? 1 : 0;
     const int my_v = lane >> (5 - lg2V);
     const bool writer = (lane & ((32 >> lg2V) - 1)) == 0;
@@ -411,7 +420,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                     if (writer) {
                         const int r = my_v / B, b = my_v % B;
                         const int lr = g + G * (t * R + r);
-                        if (lr < nrows) red[((int64_t)s * p.chunk_rows + lr) * B + b] = acc[0];
+                        if (lr < nrows) red((s * p.chunk_rows + lr) * B + b) = acc[0];
                     }
                 };
                 for (int t = 0; t < nrounds; t += 2) {
@@ -426,11 +435,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
         asm volatile("griddepcontrol.wait;" ::: "memory");
         __syncthreads();
         // fixed-order sum over spans
-        for (int i = tid; i < nrows * B; i += kThreads) {
+        for (int i = tid; i < nrows * B; i += NT) {
             const int lr = i / B, b = i % B;
             if (b >= p.B) continue;
             float sum = 0.f;
-            for (int s = 0; s < p.spans; ++s) sum += red[((int64_t)s * p.chunk_rows + lr) * B + b];
+            for (int s = 0; s < p.spans; ++s) sum += red((s * p.chunk_rows + lr) * B + b);
             store_y(item.Y, p.y_dtype, (int64_t)b * item.N + q0 + lr, sum);
         }
         __syncthreads();
@@ -441,25 +450,28 @@ struct Config {
     int bits, B, KW, R;
 };
 
-// The dynamic shared-memory opt-in is a per-device function attribute: set it
-// once per device to the largest size any launch of this instantiation uses.
-template <int BITS, int B, int KW, int R, bool F16>
+// Dynamic shared memory opt-in and a carveout that leaves room for two CTAs
+// per SM: per-device function attributes, set once per device.
+template <int BITS, int B, int KW, int R, bool F16, int NT>
 cudaError_t run(const GemvParams& p, int grid, size_t smem, cudaStream_t s)
 {
-    auto k = gemv_kernel<BITS, B, KW, R, F16>;
-    static int configured[64] = {0};
+    auto k = gemv_kernel<BITS, B, KW, R, F16, NT>;
+    static bool configured[64] = {false};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-    if (configured[dev] < (int)smem) {
+    if (!configured[dev]) {
         e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem);
         if (e != cudaSuccess) return e;
-        configured[dev] = kMaxSmem;
+        e = cudaFuncSetAttribute(k, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                 B <= 2 ? LOGQ_GEMV_CARVEOUT : (int)cudaSharedmemCarveoutMaxShared);
+        if (e != cudaSuccess) return e;
+        configured[dev] = true;
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)grid);
-    cfg.blockDim = dim3(kThreads);
+    cfg.blockDim = dim3(NT);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
@@ -471,21 +483,22 @@ cudaError_t run(const GemvParams& p, int grid, size_t smem, cudaStream_t s)
 }
 
 template <bool F16>
-cudaError_t dispatch(int bits, int Bp, const GemvParams& p, int grid, size_t smem, cudaStream_t s)
+cudaError_t dispatch(int bits, int Bp, bool large, const GemvParams& p, int grid, size_t smem, cudaStream_t s)
 {
+    constexpr int L = kLargeThreads, S = kSmallThreads;
     if (bits == 4) {
         switch (Bp) {
-        case 1: return run<4, 1, 32, 8, F16>(p, grid, smem, s);
-        case 2: return run<4, 2, 32, 4, F16>(p, grid, smem, s);
-        case 4: return run<4, 4, 16, 2, F16>(p, grid, smem, s);
-        case 8: return run<4, 8, 8, 1, F16>(p, grid, smem, s);
-        case 16: return run<4, 16, 8, 1, F16>(p, grid, smem, s);
+        case 1: return large ? run<4, 1, 32, 8, F16, L>(p, grid, smem, s) : run<4, 1, 32, 8, F16, S>(p, grid, smem, s);
+        case 2: return large ? run<4, 2, 32, 4, F16, L>(p, grid, smem, s) : run<4, 2, 32, 4, F16, S>(p, grid, smem, s);
+        case 4: return run<4, 4, 16, 2, F16, S>(p, grid, smem, s);
+        case 8: return run<4, 8, 8, 1, F16, S>(p, grid, smem, s);
+        case 16: return run<4, 16, 8, 1, F16, S>(p, grid, smem, s);
         }
     } else {
         switch (Bp) {
-        case 1: return run<3, 1, 32, 8, F16>(p, grid, smem, s);
-        case 2: return run<3, 2, 32, 4, F16>(p, grid, smem, s);
-        case 4: return run<3, 4, 32, 2, F16>(p, grid, smem, s);
+        case 1: return large ? run<3, 1, 32, 8, F16, L>(p, grid, smem, s) : run<3, 1, 32, 8, F16, S>(p, grid, smem, s);
+        case 2: return large ? run<3, 2, 32, 4, F16, L>(p, grid, smem, s) : run<3, 2, 32, 4, F16, S>(p, grid, smem, s);
+        case 4: return run<3, 4, 32, 2, F16, S>(p, grid, smem, s);
         }
     }
     return cudaErrorInvalidValue;
@@ -506,6 +519,24 @@ int kw_for(int bits, int Bp)
     return Bp <= 2 ? 32 : (Bp == 4 ? 16 : 8);
 }
 
+// The table lookups address shared memory relative to kTabOff, which is where
+// dynamic shared memory starts when a kernel has no static shared memory.
+cudaError_t check_shared_base()
+{
+    static int ok[64] = {0};   // 0 unknown, 1 yes, -1 no
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    if (ok[dev] == 0) {
+        int reserved = -1;
+        e = cudaDeviceGetAttribute(&reserved, cudaDevAttrReservedSharedMemoryPerBlock, dev);
+        if (e != cudaSuccess) return e;
+        ok[dev] = (reserved == (int)kTabOff) ? 1 : -1;
+    }
+    return ok[dev] > 0 ? cudaSuccess : cudaErrorNotSupported;
+}
+
 }  // namespace
 
 bool gemv_supports(int bits, int64_t B)
@@ -518,6 +549,8 @@ bool gemv_supports(int bits, int64_t B)
 cudaError_t launch_gemv_group(const GroupArgs& a, cudaStream_t s)
 {
     if (a.count < 1 || a.count > kMaxItems) return cudaErrorInvalidValue;
+    cudaError_t e = check_shared_base();
+    if (e != cudaSuccess) return e;
     const int Bp = padded_batch(a.B);
     const int KW = kw_for(a.bits, Bp);
     const int span = 32 * KW;
@@ -525,26 +558,34 @@ cudaError_t launch_gemv_group(const GroupArgs& a, cudaStream_t s)
     memset(&p, 0, sizeof p);
     p.nitems = a.count;
     p.X = static_cast<const uint16_t*>(a.X);
+    p.err = &a.ws->error;
     p.K = (int32_t)a.K;
     p.B = (int32_t)a.B;
     p.y_dtype = a.y_dtype;
     p.row_bytes = (a.bits == 4) ? a.K / 2 : a.K / 32 * 12;
     p.spans = (int32_t)((a.K + span - 1) / span);
-    if (p.spans >= kWarps) {
+    int64_t total_rows = 0;
+    for (int i = 0; i < a.count; ++i) total_rows += a.item[i].N;
+    // Batch 1-2: large launches one 512-thread CTA per SM, small ones one
+    // 256-thread CTA per SM.  Batch 4 and more: two 256-thread CTAs per SM.
+    const bool large = Bp <= 2 && total_rows * p.row_bytes >= kSplitBytes;
+    const int threads = large ? kLargeThreads : kSmallThreads;
+    const int per_sm = Bp >= 4 ? 2 : 1;
+    const int warps = threads / 32;
+    if (p.spans >= warps) {
         p.groups = 1;
-        p.span_cols = kWarps;
+        p.span_cols = warps;
     } else {
-        p.groups = kWarps / p.spans;
+        p.groups = warps / p.spans;
         p.span_cols = p.spans;
     }
     p.pf = static_cast<const uint8_t*>(a.pf);
     p.pf_bytes = a.pf ? a.pf_bytes : 0;
 
-    // CTAs in proportion to each matrix's rows (at least one each, at most one per row).
+    // CTAs in proportion to each matrix's rows (at least one each, at most one
+    // per row).
     const int sms = sm_count() > 0 ? sm_count() : 148;
-    int64_t total_rows = 0;
-    for (int i = 0; i < a.count; ++i) total_rows += a.item[i].N;
-    int grid = (int)(total_rows < sms ? total_rows : sms);
+    int grid = (int)(total_rows < (int64_t)sms * per_sm ? total_rows : (int64_t)sms * per_sm);
     if (grid < a.count) grid = a.count;
     int ctas[kMaxItems] = {0};
     int used = 0;
@@ -601,10 +642,10 @@ cudaError_t launch_gemv_group(const GroupArgs& a, cudaStream_t s)
     if (chunk > max_rows) chunk = max_rows;
     if (chunk < 1) return cudaErrorInvalidValue;
     p.chunk_rows = (int32_t)chunk;
-    const int nent = (a.bits == 4) ? 256 : 64;
-    const size_t smem = 65536 + (size_t)nent * kTabStride + (size_t)p.spans * chunk * Bp * 4;
-    return a.x_f16 ? dispatch<true>(a.bits, Bp, p, grid, smem, s)
-                   : dispatch<false>(a.bits, Bp, p, grid, smem, s);
+    const size_t tab = (size_t)(a.bits == 4 ? 256 : 64) * kTabStride;
+    const size_t smem = red_in_table(a.bits, Bp) ? tab : tab + (size_t)p.spans * chunk * Bp * 4;
+    return a.x_f16 ? dispatch<true>(a.bits, Bp, large, p, grid, smem, s)
+                   : dispatch<false>(a.bits, Bp, large, p, grid, smem, s);
 }
 
 cudaError_t launch_gemv(const LinearArgs& a, cudaStream_t s)

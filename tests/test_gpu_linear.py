@@ -64,6 +64,14 @@ def test_gemv_16bit_output(logq, xdt, B):
     run_case(logq, 384, 1024, 4, B, xdt, ydt=xdt, seed=3)
 
 
+@pytest.mark.parametrize("bits,N,K,B", [(4, 20491, 2048, 1), (4, 20491, 2048, 2), (3, 27403, 2048, 1),
+                                         (3, 27403, 2048, 2), (4, 5131, 8192, 1)])
+def test_gemv_large_launch(logq, bits, N, K, B):
+    """Launches above the size at which the batch-1/2 decode kernel switches to
+    one 16-warp CTA per SM (20 MiB of codes), ragged row counts."""
+    run_case(logq, N, K, bits, B, torch.bfloat16, seed=N + B + bits)
+
+
 def test_gemv_config_single_layer(logq):
     """512 x 2048 layer, fp16 x [1, 2048], b = 1.5, seed 0."""
     run_case(logq, 512, 2048, 4, 1, torch.float16, seed=0)
