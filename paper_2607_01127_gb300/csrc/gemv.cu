@@ -300,12 +300,16 @@ __global__ void __launch_bounds__(NT, 512 / NT) gemv_kernel(const __grid_constan
         const int64_t lane_byte = active ? ((BITS == 4) ? (int64_t)k0 / 2 : (int64_t)k0 / 32 * 12) : 0;
         return item.codes + (q0 + g) * p.row_bytes + lane_byte;
     };
-    auto load_round = [&](CodeVec<NW> (&c)[R], const uint8_t* first, int my_rows, int t) {
-        const int here = my_rows - t * R;
-        const uint8_t* rp = first + (int64_t)t * R * rstride;
+    // codes of the round whose first row is at rp, here = rows left from it
+    auto load_round = [&](CodeVec<NW> (&c)[R], const uint8_t* rp, int here) {
+        if (here >= R) {
 #pragma unroll
-        for (int r = 0; r < R; ++r)
-            if (r < here) c[r] = ld_codes<NW>(rp + (int64_t)r * rstride);
+            for (int r = 0; r < R; ++r) c[r] = ld_codes<NW>(rp + r * rstride);
+        } else {
+#pragma unroll
+            for (int r = 0; r < R; ++r)
+                if (r < here) c[r] = ld_codes<NW>(rp + r * rstride);
+        }
     };
     bool preloaded = false;                     // ca holds the first round of the first (chunk, span)
     {
@@ -314,7 +318,7 @@ __global__ void __launch_bounds__(NT, 512 / NT) gemv_kernel(const __grid_constan
         if (compute_warp && my_rows0 > 0 && scol < p.spans) {
             int k0;
             bool active;
-            load_round(ca, span_first(r0, scol, k0, active), my_rows0, 0);
+            load_round(ca, span_first(r0, scol, k0, active), my_rows0);
             preloaded = true;
         }
     }
@@ -374,7 +378,6 @@ __global__ void __launch_bounds__(NT, 512 / NT) gemv_kernel(const __grid_constan
         const int64_t q1 = (q0 + p.chunk_rows < r1) ? q0 + p.chunk_rows : r1;
         const int nrows = (int)(q1 - q0);
         const int my_rows = (nrows > g) ? (nrows - g + G - 1) / G : 0;
-        const int nrounds = (my_rows + R - 1) / R;
         if (compute_warp && my_rows > 0) {
             for (int s = scol; s < p.spans; s += SC) {
                 int k0;
@@ -383,7 +386,7 @@ __global__ void __launch_bounds__(NT, 512 / NT) gemv_kernel(const __grid_constan
                 // Rounds of R rows with two code buffers: the loads of round t+1 are
                 // in flight while round t is decoded.  Full rounds run unguarded;
                 // the last round guards its rows (warp-uniform branches).
-                if (!preloaded) load_round(ca, first, my_rows, 0);
+                if (!preloaded) load_round(ca, first, my_rows);
                 preloaded = false;
                 asm volatile("griddepcontrol.wait;" ::: "memory");
                 // activations for this span stay in registers (zero on idle lanes)
@@ -401,8 +404,12 @@ __global__ void __launch_bounds__(NT, 512 / NT) gemv_kernel(const __grid_constan
                         if (i + 3 < NPAIR) xr[b][i + 3] = v.w;
                     }
                 }
-                auto run_round = [&](const CodeVec<NW> (&c)[R], int t) {
-                    const int here = my_rows - t * R;
+                // the writer lane's result of each round: row my_v / B, batch
+                // row my_v % B; its local row and partial-buffer index advance
+                // by constants
+                int lr_w = g + G * (my_v / B);
+                int red_i = (s * p.chunk_rows + lr_w) * B + my_v % B;
+                auto run_round = [&](const CodeVec<NW> (&c)[R], int here) {
                     float acc[V], acc_hi[V];
 #pragma unroll
                     for (int i = 0; i < V; ++i) acc[i] = acc_hi[i] = 0.f;
@@ -417,18 +424,57 @@ __global__ void __launch_bounds__(NT, 512 / NT) gemv_kernel(const __grid_constan
 #pragma unroll
                     for (int i = 0; i < V; ++i) acc[i] += acc_hi[i];
                     reduce_scatter<V>(acc, lane);
-                    if (writer) {
-                        const int r = my_v / B, b = my_v % B;
-                        const int lr = g + G * (t * R + r);
-                        if (lr < nrows) red((s * p.chunk_rows + lr) * B + b) = acc[0];
-                    }
+                    if (writer && lr_w < nrows) red(red_i) = acc[0];
+                    lr_w += G * R;
+                    red_i += G * R * B;
                 };
-                for (int t = 0; t < nrounds; t += 2) {
-                    if (t + 1 < nrounds) load_round(cb, first, my_rows, t + 1);
-                    run_round(ca, t);
-                    if (t + 1 >= nrounds) break;
-                    if (t + 2 < nrounds) load_round(ca, first, my_rows, t + 2);
-                    run_round(cb, t + 1);
+                // rounds of R rows with two code buffers: the loads of the next
+                // round are in flight while this one is decoded
+                if constexpr (R == 1) {
+                    // one-row rounds (batches of 8 and 16): a counted loop with
+                    // indices recomputed from the round number, which keeps
+                    // fewer registers live in these register-bound kernels
+                    auto load1 = [&](CodeVec<NW> (&c)[R], int t) {
+                        if (t < my_rows) c[0] = ld_codes<NW>(first + (int64_t)t * rstride);
+                    };
+                    auto run1 = [&](const CodeVec<NW> (&c)[R], int t) {
+                        float acc[V], acc_hi[V];
+#pragma unroll
+                        for (int i = 0; i < V; ++i) acc[i] = acc_hi[i] = 0.f;
+                        if (t < my_rows) decode_row<BITS, B, NW, F16>(c[0], base_lane, xr, acc, acc_hi);
+#pragma unroll
+                        for (int i = 0; i < V; ++i) acc[i] += acc_hi[i];
+                        reduce_scatter<V>(acc, lane);
+                        if (writer) {
+                            const int lr = g + G * t;
+                            if (lr < nrows) red((s * p.chunk_rows + lr) * B + my_v % B) = acc[0];
+                        }
+                    };
+                    const int nrounds = my_rows;
+                    for (int t = 0; t < nrounds; t += 2) {
+                        load1(cb, t + 1);
+                        run1(ca, t);
+                        if (t + 1 >= nrounds) break;
+                        load1(ca, t + 2);
+                        run1(cb, t + 1);
+                    }
+                } else {
+                    const uint8_t* rp = first;
+                    int here = my_rows;               // rows of this warp from round rp on
+                    while (true) {
+                        const uint8_t* rn = rp + R * rstride;
+                        if (here > R) load_round(cb, rn, here - R);
+                        run_round(ca, here);
+                        if (here <= R) break;
+                        rp = rn;
+                        here -= R;
+                        rn = rp + R * rstride;
+                        if (here > R) load_round(ca, rn, here - R);
+                        run_round(cb, here);
+                        if (here <= R) break;
+                        rp = rn;
+                        here -= R;
+                    }
                 }
             }
         }
