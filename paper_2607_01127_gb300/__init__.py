@@ -218,6 +218,8 @@ def logq_linear(codes, cb: Codebook, X, N: int, K: int, y_dtype=None, Y=None, wo
     yd = LOGQ_F32 if y_dtype is None else (_dtype_code(y_dtype) if not isinstance(y_dtype, int) else y_dtype)
     if Y is None:
         Y = torch.empty((B, N), dtype=_torch_dtype(yd), device=X.device)
+    assert Y.dtype == _torch_dtype(yd) and Y.is_contiguous() and Y.numel() == B * N, \
+        "Y must be a contiguous [B, N] tensor of the output dtype"
     if workspace is None:
         workspace = new_workspace(X.device)
     st = _lib().logq_linear(ctypes.c_void_p(codes.data_ptr()), ctypes.byref(cb), ctypes.c_void_p(X.data_ptr()),
@@ -243,6 +245,8 @@ def logq_linear_grouped(items, X, K: int, y_dtype=None, workspace=None, prefetch
     for i, (codes, cb, N, Y) in enumerate(items):
         if Y is None:
             Y = torch.empty((B, N), dtype=_torch_dtype(yd), device=X.device)
+        assert Y.dtype == _torch_dtype(yd) and Y.is_contiguous() and Y.numel() == B * N, \
+            "Y must be a contiguous [B, N] tensor of the output dtype"
         outs.append(Y)
         keep.append(cb)
         arr[i] = LinearItem(ctypes.c_void_p(codes.data_ptr()), ctypes.pointer(cb), int(N),

@@ -18,6 +18,10 @@
 //              per lookup in a per-lane-replicated pair table, and writes the
 //              bf16 (or fp16) weight tile into shared memory in the K-major
 //              128-byte-swizzled layout the MMA reads, followed by a proxy fence.
+// The pair table starts the dynamic shared memory, at the fixed shared address
+// kTabOff, with 256-byte rows: the offset of an entry, byte << 8 | 4 * lane,
+// is one byte permute of the code word and the table base is the load's
+// immediate offset.  The code ring lives in the free upper halves of the rows.
 // Every mbarrier wait is bounded: a wait that exceeds ~1 s of clock cycles
 // raises an abort flag, records LOGQ_ERR_TIMEOUT in the caller's workspace and
 // lets every role leave its loop; the kernel drains what it issued, frees its
@@ -49,7 +53,12 @@ constexpr int kXStageBytes = kBN * kBK * 2;      // 32 KiB
 constexpr int kWStageBytes = kBM * kBK * 2;      // 16 KiB
 constexpr int kCodeSlotBytes = 16;               // codes of half a row and stage (<= 16 B)
 constexpr int kCodeStageBytes = kDecodeThreads * kCodeSlotBytes;
-constexpr int kTabBytes4 = 256 * 128;            // 4-bit pair table, 32 copies
+// Shared address at which dynamic shared memory starts in a kernel without
+// static shared memory (the per-CTA reserved area comes first).
+constexpr uint32_t kTabOff = 1024;
+constexpr uint32_t kTabRow = 256;                // 32 lane copies in the first 128 bytes
+constexpr uint32_t kTabRegion = 256 * kTabRow;   // table rows (the 4-bit table uses all 256)
+static_assert(kCodeRing * kCodeStageBytes <= 256 * 128, "code ring must fit in the table rows' free halves");
 constexpr uint32_t kTmemCols = 2 * kBN;          // two fp32 accumulators
 constexpr long long kWaitLimit = 2000000000LL;   // cycles (~1 s)
 
@@ -226,11 +235,19 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32])
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
-__device__ __forceinline__ uint32_t lds32(uint32_t addr)
+// Pair-table entry at byte offset off from the table base.
+__device__ __forceinline__ uint32_t lds_tab(uint32_t off)
 {
     uint32_t v;
-    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr));
+    asm volatile("ld.shared.u32 %0, [%1+%2];" : "=r"(v) : "r"(off), "n"(kTabOff));
     return v;
+}
+
+__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel)
+{
+    uint32_t r;
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(r) : "r"(a), "r"(b), "r"(sel));
+    return r;
 }
 
 __device__ __forceinline__ uint4 lds128(uint32_t addr)
@@ -252,26 +269,26 @@ __global__ void __launch_bounds__(kThreads, 1)
 prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ CUtensorMap xmap)
 {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
-    // Layout: the pair table sits at the first 32 KiB-aligned shared address
-    // (so a lookup address is an OR of fields); the code ring and barriers use
-    // the space below it when it is large enough, else they follow the stages.
-    //   [code ring | barriers | pad] table (32 KiB) | X stages | W stages [| code ring | barriers]
+    // Layout: pair table (code ring in its rows' free halves) | X stages | W stages | barriers
     const uint32_t sbase = smem_u32(smem_raw);
-    const uint32_t tab = (sbase + 32767u) & ~32767u;
-    const uint32_t xs0 = tab + kTabBytes4;
+    const uint32_t xs0 = sbase + kTabRegion;
     const uint32_t ws0 = xs0 + kXStages * kXStageBytes;
-    constexpr uint32_t kLowBytes = kCodeRing * kCodeStageBytes + 256;
-    const bool low = tab - sbase >= kLowBytes;
-    const uint32_t cr0 = low ? sbase : ws0 + kWStages * kWStageBytes;
-    const uint32_t bar0 = cr0 + kCodeRing * kCodeStageBytes;
-    const uint32_t layout_end = low ? ws0 + kWStages * kWStageBytes : bar0 + 256;
-    if (layout_end > sbase + p.smem_bytes) {          // launch too small for this layout: refuse
+    const uint32_t bar0 = ws0 + kWStages * kWStageBytes;
+    const uint32_t layout_end = bar0 + 256;
+    // the lookups address the table as an offset from kTabOff; refuse a launch
+    // whose shared window differs or is too small for this layout
+    if (sbase != kTabOff || layout_end > sbase + p.smem_bytes) {
         if (threadIdx.x == 0) {
             atomicExch(&p.ws->detail, (uint32_t)kWaitLayout);
             atomicExch(&p.ws->error, (uint32_t)LOGQ_ERR_TIMEOUT);
         }
         return;
     }
+    // code-ring slot of decode thread d in ring stage g: 16 bytes in the free
+    // half of table row g * 32 + d / 8
+    auto ring_slot = [&](int g, int d) -> uint32_t {
+        return sbase + (uint32_t)(g * (kDecodeThreads / 8) + (d >> 3)) * kTabRow + 128u + ((uint32_t)(d & 7) << 4);
+    };
     uint8_t* gen = smem_raw - sbase;                  // generic pointer = gen + shared address
     // barriers: xfull[X], xempty[X], wfull[W], wempty[W], accfull[2], accempty[2], drain,
     // then the tmem slot and the abort flag
@@ -313,7 +330,7 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
             const uint32_t lo = (p.bits == 4) ? (e & 15) : (e & 7);
             const uint32_t hi = (p.bits == 4) ? (e >> 4) : (e >> 3);
             const uint32_t v = (p.lvl16[lo] & 0xffffu) | (p.lvl16[hi] << 16);
-            sts128(tab + e * 128 + part * 16, v, v, v, v);
+            sts128(sbase + e * kTabRow + part * 16, v, v, v, v);
         }
     }
     if (warp == 1) {
@@ -476,7 +493,7 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         const int d = tid - 6 * 32;                     // 0 .. kDecodeThreads-1
         const int r = d & (kBM - 1);                    // weight row within the tile
         const int h = d >> 7;                           // half: k 32h .. 32h+31 of the stage
-        const uint32_t tl = tab | (4u * (uint32_t)lane);
+        const uint32_t lane4 = 4u * (uint32_t)lane;
         const int hbytes = (p.bits == 4) ? 16 : 12;     // codes of one half row per stage
         int stage = 0;
         uint32_t phase = 0;
@@ -505,7 +522,7 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         auto issue = [&](int g) {
             if (g < total && ahead.valid) {
                 const uint8_t* src = ahead.row + (int64_t)ahead.ks * (2 * hbytes);
-                const uint32_t dst = cr0 + (g % kCodeRing) * kCodeStageBytes + d * kCodeSlotBytes;
+                const uint32_t dst = ring_slot(g % kCodeRing, d);
                 if (p.bits == 4) {
                     cp_async_16(dst, src);
                 } else {
@@ -520,51 +537,58 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         // Resolve the codes of one stage (its slot in the ring) into 16 pair values.
         auto resolve = [&](int slot, bool valid, uint32_t (&pr)[16]) {
             uint4 cv = make_uint4(0, 0, 0, 0);
-            if (valid) cv = lds128(cr0 + slot * kCodeStageBytes + d * kCodeSlotBytes);
+            if (valid) cv = lds128(ring_slot(slot, d));
             const uint32_t cw[4] = {cv.x, cv.y, cv.z, cv.w};
             if (p.bits == 4) {
                 // word i holds k = 32h + 8i .. +7 -> 16-byte chunk 4h + i of the row
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                     const uint32_t c = cw[i];
-                    pr[4 * i + 0] = lds32(((c << 7) & 0x7f80u) | tl);
-                    pr[4 * i + 1] = lds32(((c >> 1) & 0x7f80u) | tl);
-                    pr[4 * i + 2] = lds32(((c >> 9) & 0x7f80u) | tl);
-                    pr[4 * i + 3] = lds32(((c >> 17) & 0x7f80u) | tl);
+                    pr[4 * i + 0] = lds_tab(prmt(c, lane4, 0x7604u));
+                    pr[4 * i + 1] = lds_tab(prmt(c, lane4, 0x7614u));
+                    pr[4 * i + 2] = lds_tab(prmt(c, lane4, 0x7624u));
+                    pr[4 * i + 3] = lds_tab(prmt(c, lane4, 0x7634u));
                 }
             } else {
                 // one 12-byte group of 32 k; pair p -> chunk 4h + p / 4
 #pragma unroll
                 for (int i = 0; i < 3; ++i) {
-                    pr[5 * i + 0] = lds32(((cw[i] << 7) & 0x1f80u) | tl);
-                    pr[5 * i + 1] = lds32(((cw[i] << 1) & 0x1f80u) | tl);
-                    pr[5 * i + 2] = lds32(((cw[i] >> 5) & 0x1f80u) | tl);
-                    pr[5 * i + 3] = lds32(((cw[i] >> 11) & 0x1f80u) | tl);
-                    pr[5 * i + 4] = lds32(((cw[i] >> 17) & 0x1f80u) | tl);
+                    pr[5 * i + 0] = lds_tab(((cw[i] << 8) & 0x3f00u) | lane4);
+                    pr[5 * i + 1] = lds_tab(((cw[i] << 2) & 0x3f00u) | lane4);
+                    pr[5 * i + 2] = lds_tab(((cw[i] >> 4) & 0x3f00u) | lane4);
+                    pr[5 * i + 3] = lds_tab(((cw[i] >> 10) & 0x3f00u) | lane4);
+                    pr[5 * i + 4] = lds_tab(((cw[i] >> 16) & 0x3f00u) | lane4);
                 }
-                pr[15] = lds32(((cw[0] >> 23) & 0x0180u) | ((cw[1] >> 21) & 0x0600u) | ((cw[2] >> 19) & 0x1800u) | tl);
+                pr[15] = lds_tab(((cw[0] >> 22) & 0x0300u) | ((cw[1] >> 20) & 0x0c00u) | ((cw[2] >> 18) & 0x3000u) | lane4);
             }
         };
         // Software pipeline: the pairs of stage g+1 are looked up while stage g
         // waits for its weight slot and is stored.
         for (int g = 0; g < kCodeRing - 1; ++g) issue(g);
-        uint32_t cur_pr[16], next_pr[16];
+        uint32_t pr_a[16], pr_b[16];
         int slot = 0;                                   // ring slot of stage g
         if (total > 0) {
             issue(kCodeRing - 1);
             cp_async_wait<kCodeRing - 1>();
-            resolve(slot, cur.valid, cur_pr);
+            resolve(slot, cur.valid, pr_a);
             step(cur);
         }
-        for (int g = 0; g < total; ++g) {
+        // One stage: look up the next stage's pairs into nxt, then store this
+        // stage's (cur) once its weight slot is free.  Called with the two
+        // buffers in alternating roles, so no pairs are copied.
+        bool ok = true;
+        auto stage_step = [&](int g, const uint32_t (&cur_pr)[16], uint32_t (&nxt_pr)[16]) {
             if (++slot == kCodeRing) slot = 0;
             if (g + 1 < total) {
                 issue(g + kCodeRing);
                 cp_async_wait<kCodeRing - 1>();
-                resolve(slot, cur.valid, next_pr);
+                resolve(slot, cur.valid, nxt_pr);
                 step(cur);
             }
-            if (!warp_wait(wempty(stage), phase ^ 1u, abort_flag, p.ws, kWaitDecode)) break;
+            if (!warp_wait(wempty(stage), phase ^ 1u, abort_flag, p.ws, kWaitDecode)) {
+                ok = false;
+                return;
+            }
             const uint32_t wrow = ws0 + stage * kWStageBytes + r * 128;
             const uint32_t sw = (uint32_t)(r & 7);
 #pragma unroll
@@ -575,8 +599,11 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
             __syncwarp();
             if (lane == 0) mbar_arrive(wfull(stage));
             if (++stage == kWStages) { stage = 0; phase ^= 1u; }
-#pragma unroll
-            for (int i = 0; i < 16; ++i) cur_pr[i] = next_pr[i];
+        };
+        for (int g = 0; g < total && ok; g += 2) {
+            stage_step(g, pr_a, pr_b);
+            if (g + 1 >= total || !ok) break;
+            stage_step(g + 1, pr_b, pr_a);
         }
         cp_async_wait<0>();
     }
@@ -625,16 +652,8 @@ uint32_t make_idesc(bool f16_inputs)
     return d;
 }
 
-constexpr uint32_t kStageRegion = kXStages * kXStageBytes + kWStages * kWStageBytes;
-constexpr uint32_t kRingRegion = kCodeRing * kCodeStageBytes + 256;
-
-// Dynamic shared memory for the layout above, given where the dynamic region
-// starts in the CTA's shared window (after the reserved shared memory).
-uint32_t smem_bytes_for(uint32_t start)
-{
-    const uint32_t pad = (32768u - (start & 32767u)) & 32767u;
-    return pad >= kRingRegion ? pad + kTabBytes4 + kStageRegion : pad + kTabBytes4 + kStageRegion + kRingRegion;
-}
+// Dynamic shared memory of the layout: table rows, X and W stages, barriers.
+constexpr uint32_t kSmemBytes = kTabRegion + kXStages * kXStageBytes + kWStages * kWStageBytes + 256;
 
 }  // namespace
 
@@ -682,8 +701,8 @@ cudaError_t launch_prefill(const LinearArgs& a, cudaStream_t s)
         int reserved = 0, optin = 0;
         if ((e = cudaDeviceGetAttribute(&reserved, cudaDevAttrReservedSharedMemoryPerBlock, dev)) != cudaSuccess) return e;
         if ((e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev)) != cudaSuccess) return e;
-        const uint32_t bytes = smem_bytes_for((uint32_t)reserved);
-        if (bytes > (uint32_t)optin) return cudaErrorNotSupported;
+        const uint32_t bytes = kSmemBytes;
+        if (reserved != (int)kTabOff || bytes > (uint32_t)optin) return cudaErrorNotSupported;
         e = cudaFuncSetAttribute(prefill_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
         if (e != cudaSuccess) return e;
         configured[dev] = bytes;
