@@ -60,6 +60,13 @@ constexpr int kMaxItems = 4;
 #define LOGQ_GEMV_SPLIT_BYTES (20 << 20)
 #endif
 constexpr int64_t kSplitBytes = LOGQ_GEMV_SPLIT_BYTES;
+// Batch-1 4-bit launches below this many bytes of codes take 16 k per lane
+// (twice the spans, half the activations per lane): their few rows per warp
+// finish sooner after the activations arrive.
+#ifndef LOGQ_GEMV_TINY_BYTES
+#define LOGQ_GEMV_TINY_BYTES (4 << 20)
+#endif
+constexpr int64_t kTinyBytes = LOGQ_GEMV_TINY_BYTES;
 // Shared-memory carveout of the batch-1/2 decode kernels, in percent of the
 // maximum: 58 % is 132 KiB, room for two CTAs of 64 KiB (plus their reserved
 // 1 KiB).  The rest of the 256 KiB per SM is L1, which also holds the data of
@@ -529,12 +536,15 @@ cudaError_t run(const GemvParams& p, int grid, size_t smem, cudaStream_t s)
 }
 
 template <bool F16>
-cudaError_t dispatch(int bits, int Bp, bool large, const GemvParams& p, int grid, size_t smem, cudaStream_t s)
+cudaError_t dispatch(int bits, int Bp, bool large, bool tiny, const GemvParams& p, int grid, size_t smem,
+                     cudaStream_t s)
 {
     constexpr int L = kLargeThreads, S = kSmallThreads;
     if (bits == 4) {
         switch (Bp) {
-        case 1: return large ? run<4, 1, 32, 8, F16, L>(p, grid, smem, s) : run<4, 1, 32, 8, F16, S>(p, grid, smem, s);
+        case 1:
+            if (large) return run<4, 1, 32, 8, F16, L>(p, grid, smem, s);
+            return tiny ? run<4, 1, 16, 8, F16, S>(p, grid, smem, s) : run<4, 1, 32, 8, F16, S>(p, grid, smem, s);
         case 2: return large ? run<4, 2, 32, 4, F16, L>(p, grid, smem, s) : run<4, 2, 32, 4, F16, S>(p, grid, smem, s);
         case 4: return run<4, 4, 16, 2, F16, S>(p, grid, smem, s);
         case 8: return run<4, 8, 8, 1, F16, S>(p, grid, smem, s);
@@ -559,9 +569,10 @@ int padded_batch(int64_t B)
     return 16;
 }
 
-int kw_for(int bits, int Bp)
+int kw_for(int bits, int Bp, bool tiny)
 {
     if (bits == 3) return 32;
+    if (Bp == 1 && tiny) return 16;
     return Bp <= 2 ? 32 : (Bp == 4 ? 16 : 8);
 }
 
@@ -598,7 +609,11 @@ cudaError_t launch_gemv_group(const GroupArgs& a, cudaStream_t s)
     cudaError_t e = check_shared_base();
     if (e != cudaSuccess) return e;
     const int Bp = padded_batch(a.B);
-    const int KW = kw_for(a.bits, Bp);
+    int64_t total_rows = 0;
+    for (int i = 0; i < a.count; ++i) total_rows += a.item[i].N;
+    const int64_t row_bytes = (a.bits == 4) ? a.K / 2 : a.K / 32 * 12;
+    const bool tiny = a.bits == 4 && Bp == 1 && total_rows * row_bytes < kTinyBytes;
+    const int KW = kw_for(a.bits, Bp, tiny);
     const int span = 32 * KW;
     GemvParams p;
     memset(&p, 0, sizeof p);
@@ -608,10 +623,8 @@ cudaError_t launch_gemv_group(const GroupArgs& a, cudaStream_t s)
     p.K = (int32_t)a.K;
     p.B = (int32_t)a.B;
     p.y_dtype = a.y_dtype;
-    p.row_bytes = (a.bits == 4) ? a.K / 2 : a.K / 32 * 12;
+    p.row_bytes = row_bytes;
     p.spans = (int32_t)((a.K + span - 1) / span);
-    int64_t total_rows = 0;
-    for (int i = 0; i < a.count; ++i) total_rows += a.item[i].N;
     // Batch 1-2: large launches one 512-thread CTA per SM, small ones one
     // 256-thread CTA per SM.  Batch 4 and more: two 256-thread CTAs per SM.
     const bool large = Bp <= 2 && total_rows * p.row_bytes >= kSplitBytes;
@@ -690,8 +703,8 @@ cudaError_t launch_gemv_group(const GroupArgs& a, cudaStream_t s)
     p.chunk_rows = (int32_t)chunk;
     const size_t tab = (size_t)(a.bits == 4 ? 256 : 64) * kTabStride;
     const size_t smem = red_in_table(a.bits, Bp) ? tab : tab + (size_t)p.spans * chunk * Bp * 4;
-    return a.x_f16 ? dispatch<true>(a.bits, Bp, large, p, grid, smem, s)
-                   : dispatch<false>(a.bits, Bp, large, p, grid, smem, s);
+    return a.x_f16 ? dispatch<true>(a.bits, Bp, large, tiny, p, grid, smem, s)
+                   : dispatch<false>(a.bits, Bp, large, tiny, p, grid, smem, s);
 }
 
 cudaError_t launch_gemv(const LinearArgs& a, cudaStream_t s)
