@@ -452,7 +452,7 @@ def run_ours(args):
         "gpu_launches": launches_per_step * args.steps,
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": pk["hbm_gbs"], "unit": "GB/s",
                      "frac": round(achieved / pk["hbm_gbs"], 4), "peak_source": pk_kind,
-                     "traffic": tr, "kernel": "gemv_kernel<4,1,32,8,bf16>",
+                     "traffic": tr, "kernel": "gemv_kernel, batch 1, 4-bit (16 k per lane for q/k/v and o, 32 for gate/up and down)",
                      "algorithmic_bytes_per_launch": round(gemv_bytes_per_launch, 1),
                      "frac_of_8TBs": round(achieved / 8000.0, 4)},
         "clocks": clocks.summary(),

@@ -72,6 +72,13 @@ def test_gemv_large_launch(logq, bits, N, K, B):
     run_case(logq, N, K, bits, B, torch.bfloat16, seed=N + B + bits)
 
 
+@pytest.mark.parametrize("N,K", [(4095, 2048), (4096, 2048), (20479, 2048), (20480, 2048)])
+def test_gemv_launch_shape_boundaries(logq, N, K):
+    """Batch-1 launches on either side of the sizes where the decode kernel
+    changes shape (4 MiB and 20 MiB of codes)."""
+    run_case(logq, N, K, 4, 1, torch.bfloat16, seed=N)
+
+
 def test_gemv_config_single_layer(logq):
     """512 x 2048 layer, fp16 x [1, 2048], b = 1.5, seed 0."""
     run_case(logq, 512, 2048, 4, 1, torch.float16, seed=0)
