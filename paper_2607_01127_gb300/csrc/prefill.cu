@@ -4,20 +4,27 @@
 // dense bf16/fp16 contraction).
 //
 // One persistent CTA per SM walks 128 (weights) x 256 (tokens) output tiles.
+// The dequantised weight tile (the MMA's A operand) lives in tensor memory, not
+// in shared memory: tensor memory holds one fp32 accumulator (256 columns) and
+// eight weight stages (32 columns each), and shared memory holds the pair table
+// and five X stages.
 // Warp roles:
 //   warp 0     TMA producer: X tiles [256 tokens x 64 k] with 128-byte swizzle.
 //   warp 1     MMA issuer: tcgen05.mma kind::f16, M = 128 (weight rows),
-//              N = 256 (tokens), K = 16, fp32 accumulators in tensor memory,
-//              double-buffered (2 x 256 columns), so the epilogue of one tile
-//              overlaps the main loop of the next.  Also allocates TMEM.
-//   warps 2-5  epilogue: tcgen05.ld of the accumulator, stores of Y (each warp
-//              reads its TMEM lane quarter; lane n writes Y[t][n0 + n]).
-//   warps 6-13 decode: two threads per weight row of the tile, each owning 32
+//              N = 256 (tokens), K = 16, A from tensor memory, B (X) from
+//              shared memory, fp32 accumulator in tensor memory.  Also
+//              allocates TMEM.
+//   warps 2-9  epilogue: two warps per TMEM lane quarter, each draining 128
+//              token columns with tcgen05.ld; 16-bit outputs are rounded into
+//              registers and the accumulator is handed back before the stores
+//              of Y (lane n writes Y[t][n0 + n]).
+//   warps 10-17 decode: two threads per weight row of the tile, each owning 32
 //              of the stage's 64 k; a thread streams its codes into its own
 //              16-byte slot of a shared ring with cp.async, resolves two codes
 //              per lookup in a per-lane-replicated pair table, and writes the
-//              bf16 (or fp16) weight tile into shared memory in the K-major
-//              128-byte-swizzled layout the MMA reads, followed by a proxy fence.
+//              16 bf16 (or fp16) pairs to its row's TMEM lane with tcgen05.st.
+//              tcgen05.st reaches only the warp's lane quarter (warp % 4), so a
+//              thread's weight row is 32 * (warp % 4) + lane.
 // The pair table starts the dynamic shared memory, at the fixed shared address
 // kTabOff, with 256-byte rows: the offset of an entry, byte << 8 | 4 * lane,
 // is one byte permute of the code word and the table base is the load's
@@ -43,14 +50,15 @@ namespace {
 constexpr int kBM = 128;                 // weight rows per tile (MMA M)
 constexpr int kBN = 256;                 // tokens per tile (MMA N)
 constexpr int kBK = 64;                  // k per stage (one 128-byte swizzle atom of bf16)
-constexpr int kXStages = 3;              // X tiles in flight (TMA)
-constexpr int kWStages = 4;              // dequantised weight tiles in flight (decode warps)
+constexpr int kXStages = 5;              // X tiles in flight (TMA)
+constexpr int kWStages = 8;              // dequantised weight tiles in flight (tensor memory)
 constexpr int kCodeRing = 7;             // code stages in flight per decode thread
 constexpr int kDecodeWarps = 8;
 constexpr int kDecodeThreads = 32 * kDecodeWarps;  // two threads per weight row
-constexpr int kThreads = 32 * (6 + kDecodeWarps);  // producer, MMA, 4 epilogue, decode
+constexpr int kEpiWarps = 8;                       // two per TMEM lane quarter
+constexpr int kEpi0 = 2, kDec0 = kEpi0 + kEpiWarps;  // first epilogue / decode warp
+constexpr int kThreads = 32 * (kDec0 + kDecodeWarps);  // producer, MMA, epilogue, decode
 constexpr int kXStageBytes = kBN * kBK * 2;      // 32 KiB
-constexpr int kWStageBytes = kBM * kBK * 2;      // 16 KiB
 constexpr int kCodeSlotBytes = 16;               // codes of half a row and stage (<= 16 B)
 constexpr int kCodeStageBytes = kDecodeThreads * kCodeSlotBytes;
 // Shared address at which dynamic shared memory starts in a kernel without
@@ -59,7 +67,10 @@ constexpr uint32_t kTabOff = 1024;
 constexpr uint32_t kTabRow = 256;                // 32 lane copies in the first 128 bytes
 constexpr uint32_t kTabRegion = 256 * kTabRow;   // table rows (the 4-bit table uses all 256)
 static_assert(kCodeRing * kCodeStageBytes <= 256 * 128, "code ring must fit in the table rows' free halves");
-constexpr uint32_t kTmemCols = 2 * kBN;          // two fp32 accumulators
+constexpr uint32_t kTmemCols = 512;              // accumulator (256) + weight stages (8 x 32)
+constexpr uint32_t kWCol0 = kBN;                 // first column of weight stage 0
+constexpr uint32_t kWStageCols = kBK / 2;        // 64 k of 16-bit values = 32 columns
+static_assert(kWCol0 + kWStages * kWStageCols <= kTmemCols, "weight stages must fit in tensor memory");
 constexpr long long kWaitLimit = 2000000000LL;   // cycles (~1 s)
 
 // error detail codes (workspace->detail)
@@ -185,8 +196,6 @@ __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commi
 template <int N>
 __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
 
-__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
-
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
@@ -203,16 +212,30 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t addr)
     return d;
 }
 
-__device__ __forceinline__ void mma_f16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
-                                        uint32_t accumulate)
+// A (weights) from tensor memory: row m in lane m, 16-bit k-pairs packed per column.
+__device__ __forceinline__ void mma_f16_ta(uint32_t tmem_d, uint32_t tmem_a, uint64_t bdesc, uint32_t idesc,
+                                           uint32_t accumulate)
 {
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
         "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
-        ::"r"(tmem_d), "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}"
+        ::"r"(tmem_d), "r"(tmem_a), "l"(bdesc), "r"(idesc), "r"(accumulate)
         : "memory");
 }
+
+// 16 consecutive columns of this warp's 32 TMEM lanes (lane i of the warp -> TMEM lane base + i).
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&v)[16])
+{
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+        "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};"
+        ::"r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
+          "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
+        : "memory");
+}
+
+__device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
 __device__ __forceinline__ void mma_commit(uint32_t bar)
 {
@@ -269,11 +292,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ CUtensorMap xmap)
 {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
-    // Layout: pair table (code ring in its rows' free halves) | X stages | W stages | barriers
+    // Layout: pair table (code ring in its rows' free halves) | X stages | barriers
     const uint32_t sbase = smem_u32(smem_raw);
     const uint32_t xs0 = sbase + kTabRegion;
-    const uint32_t ws0 = xs0 + kXStages * kXStageBytes;
-    const uint32_t bar0 = ws0 + kWStages * kWStageBytes;
+    const uint32_t bar0 = xs0 + kXStages * kXStageBytes;
     const uint32_t layout_end = bar0 + 256;
     // the lookups address the table as an offset from kTabOff; refuse a launch
     // whose shared window differs or is too small for this layout
@@ -290,17 +312,18 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         return sbase + (uint32_t)(g * (kDecodeThreads / 8) + (d >> 3)) * kTabRow + 128u + ((uint32_t)(d & 7) << 4);
     };
     uint8_t* gen = smem_raw - sbase;                  // generic pointer = gen + shared address
-    // barriers: xfull[X], xempty[X], wfull[W], wempty[W], accfull[2], accempty[2], drain,
+    // barriers: xfull[X], xempty[X], wfull[W], wempty[W], accfull, accempty, drain,
     // then the tmem slot and the abort flag
     auto xfull = [&](int s) { return bar0 + 8u * s; };
     auto xempty = [&](int s) { return bar0 + 8u * (kXStages + s); };
     auto wfull = [&](int s) { return bar0 + 8u * (2 * kXStages + s); };
     auto wempty = [&](int s) { return bar0 + 8u * (2 * kXStages + kWStages + s); };
     constexpr int kB0 = 2 * kXStages + 2 * kWStages;
-    auto accfull = [&](int b) { return bar0 + 8u * (kB0 + b); };
-    auto accempty = [&](int b) { return bar0 + 8u * (kB0 + 2 + b); };
-    const uint32_t drainb = bar0 + 8u * (kB0 + 4);
-    const uint32_t tmem_slot = bar0 + 8u * (kB0 + 5);
+    const uint32_t accfull = bar0 + 8u * kB0;
+    const uint32_t accempty = bar0 + 8u * (kB0 + 1);
+    const uint32_t drainb = bar0 + 8u * (kB0 + 2);
+    const uint32_t tmem_slot = bar0 + 8u * (kB0 + 3);
+    static_assert(8 * (2 * kXStages + 2 * kWStages + 3) + 8 + 4 <= 256, "barrier block overflows");
     volatile int* abort_flag = reinterpret_cast<volatile int*>(gen + tmem_slot + 8);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -313,10 +336,8 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
             mbar_init(wfull(s), kDecodeWarps);
             mbar_init(wempty(s), 1);
         }
-        for (int b = 0; b < 2; ++b) {
-            mbar_init(accfull(b), 1);
-            mbar_init(accempty(b), 4);
-        }
+        mbar_init(accfull, 1);
+        mbar_init(accempty, kEpiWarps);
         mbar_init(drainb, 1);
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -402,11 +423,10 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         bool ok = true;
         int it = 0;
         for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
-            const int buf = it & 1;
-            const uint32_t acc_phase = ((uint32_t)it >> 1) & 1u;
-            if (!warp_wait(accempty(buf), acc_phase ^ 1u, abort_flag, p.ws, kWaitMma)) break;
+            // one accumulator: the epilogue has read the previous tile's out of it
+            if (!warp_wait(accempty, ((uint32_t)it & 1u) ^ 1u, abort_flag, p.ws, kWaitMma)) break;
             tc_fence_after();
-            const uint32_t dcol = tmem_base + (uint32_t)(buf * kBN);
+            const uint32_t dcol = tmem_base;
             for (int ks = 0; ks < ksteps; ++ks) {
                 if (!warp_wait(xfull(xs), xph, abort_flag, p.ws, kWaitMma) ||
                     !warp_wait(wfull(wsg), wph, abort_flag, p.ws, kWaitMma)) {
@@ -414,13 +434,14 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
                     break;
                 }
                 tc_fence_after();
-                const uint64_t adesc = smem_desc_sw128(ws0 + wsg * kWStageBytes);
+                const uint32_t acol = tmem_base + kWCol0 + (uint32_t)wsg * kWStageCols;
                 const uint64_t bdesc = smem_desc_sw128(xs0 + xs * kXStageBytes);
                 if (elect_one()) {
 #pragma unroll
                     for (int kk = 0; kk < kBK / 16; ++kk) {
-                        // 16 k of bf16 = 32 bytes (2 descriptor units) further inside the swizzle atom
-                        mma_f16(dcol, adesc + 2 * kk, bdesc + 2 * kk, p.idesc, (ks | kk) != 0);
+                        // 16 k: 8 columns of A further on; 32 bytes (2 descriptor units)
+                        // further inside B's swizzle atom
+                        mma_f16_ta(dcol, acol + 8 * kk, bdesc + 2 * kk, p.idesc, (ks | kk) != 0);
                     }
                     mma_commit(xempty(xs));
                     mma_commit(wempty(wsg));
@@ -430,69 +451,93 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
                 if (++wsg == kWStages) { wsg = 0; wph ^= 1u; }
             }
             if (ok) {
-                if (elect_one()) mma_commit(accfull(buf));
+                if (elect_one()) mma_commit(accfull);
                 __syncwarp();
             }
         }
-    } else if (warp >= 2 && warp < 6) {
+    } else if (warp >= kEpi0 && warp < kDec0) {
         // ---------------- epilogue ----------------
+        // Two warps per TMEM lane quarter, each owning 128 of the tile's 256 token
+        // columns.  16-bit outputs are read out of tensor memory and rounded into
+        // registers first, so the accumulator is handed back before the stores.
         const int quarter = warp & 3;                   // TMEM lanes 32*quarter .. +31
+        const int ehalf = (warp - kEpi0) >> 2;          // token columns 128*ehalf .. +127
         const int row = quarter * 32 + lane;
+        const uint32_t tq = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(ehalf * 128);
         int it = 0;
         for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
-            const int buf = it & 1;
-            const uint32_t acc_phase = ((uint32_t)it >> 1) & 1u;
-            if (!warp_wait(accfull(buf), acc_phase, abort_flag, p.ws, kWaitEpilogue)) break;
+            if (!warp_wait(accfull, (uint32_t)it & 1u, abort_flag, p.ws, kWaitEpilogue)) break;
             tc_fence_after();
             const int64_t n = (int64_t)(tile % p.n_tiles_n) * kBM + row;
-            const int t0 = (tile / p.n_tiles_n) * kBN;
+            const int tb0 = (tile / p.n_tiles_n) * kBN + ehalf * 128;
+            const int jmax = (p.B - tb0) < 128 ? (p.B - tb0) : 128;   // tokens of this half (may be <= 0)
+            if (p.y_dtype == LOGQ_F32) {
 #pragma unroll 1
-            for (int c = 0; c < kBN / 32; ++c) {
-                uint32_t v[32];
-                tmem_ld32(tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * kBN + c * 32), v);
-                if (n < p.N) {
-                    // lanes hold consecutive n: each store instruction writes one
-                    // contiguous run of Y[t][n0 .. n0+31]
-                    const int tb = t0 + c * 32;
-                    const int jmax = (p.B - tb) < 32 ? (p.B - tb) : 32;
-                    const int64_t base = (int64_t)tb * p.N + n;
-                    if (p.y_dtype == LOGQ_F32) {
-                        float* y = static_cast<float*>(p.Y) + base;
-                        if (jmax == 32) {
-#pragma unroll
-                            for (int j = 0; j < 32; ++j) y[(int64_t)j * p.N] = __uint_as_float(v[j]);
-                        } else {
-#pragma unroll
-                            for (int j = 0; j < 32; ++j)
-                                if (j < jmax) y[(int64_t)j * p.N] = __uint_as_float(v[j]);
-                        }
-                    } else if (p.y_dtype == LOGQ_BF16) {
-                        __nv_bfloat16* y = static_cast<__nv_bfloat16*>(p.Y) + base;
-                        if (jmax == 32) {
-#pragma unroll
-                            for (int j = 0; j < 32; ++j) y[(int64_t)j * p.N] = __float2bfloat16_rn(__uint_as_float(v[j]));
-                        } else {
-#pragma unroll
-                            for (int j = 0; j < 32; ++j)
-                                if (j < jmax) y[(int64_t)j * p.N] = __float2bfloat16_rn(__uint_as_float(v[j]));
-                        }
-                    } else {
-                        __half* y = static_cast<__half*>(p.Y) + base;
+                for (int c = 0; c < 4; ++c) {
+                    uint32_t v[32];
+                    tmem_ld32(tq + (uint32_t)(c * 32), v);
+                    const int jm = jmax - 32 * c;
+                    if (n < p.N && jm > 0) {
+                        float* y = static_cast<float*>(p.Y) + (int64_t)(tb0 + 32 * c) * p.N + n;
 #pragma unroll
                         for (int j = 0; j < 32; ++j)
-                            if (j < jmax) y[(int64_t)j * p.N] = __float2half_rn(__uint_as_float(v[j]));
+                            if (j < jm) y[(int64_t)j * p.N] = __uint_as_float(v[j]);
+                    }
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(accempty);
+            } else {
+                const bool bf = p.y_dtype == LOGQ_BF16;
+                uint32_t pk[64];                        // tokens 2j, 2j+1 rounded to 16 bits
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    uint32_t v[32];
+                    tmem_ld32(tq + (uint32_t)(c * 32), v);
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) {
+                        const float a = __uint_as_float(v[2 * j]), b = __uint_as_float(v[2 * j + 1]);
+                        if (bf) {
+                            const __nv_bfloat162 h2 = __floats2bfloat162_rn(a, b);
+                            pk[16 * c + j] = *reinterpret_cast<const uint32_t*>(&h2);
+                        } else {
+                            const __half2 h2 = __floats2half2_rn(a, b);
+                            pk[16 * c + j] = *reinterpret_cast<const uint32_t*>(&h2);
+                        }
+                    }
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(accempty);
+                if (n < p.N && jmax > 0) {
+                    // lanes hold consecutive n: each store instruction writes one
+                    // contiguous run of Y[t][n0 .. n0+31]
+                    uint16_t* y = static_cast<uint16_t*>(p.Y) + (int64_t)tb0 * p.N + n;
+                    if (jmax == 128) {
+#pragma unroll
+                        for (int j = 0; j < 64; ++j) {
+                            y[(int64_t)(2 * j) * p.N] = (uint16_t)(pk[j] & 0xffffu);
+                            y[(int64_t)(2 * j + 1) * p.N] = (uint16_t)(pk[j] >> 16);
+                        }
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < 64; ++j) {
+                            if (2 * j < jmax) y[(int64_t)(2 * j) * p.N] = (uint16_t)(pk[j] & 0xffffu);
+                            if (2 * j + 1 < jmax) y[(int64_t)(2 * j + 1) * p.N] = (uint16_t)(pk[j] >> 16);
+                        }
                     }
                 }
             }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(accempty(buf));
         }
     } else {
         // ---------------- decode ----------------
-        const int d = tid - 6 * 32;                     // 0 .. kDecodeThreads-1
-        const int r = d & (kBM - 1);                    // weight row within the tile
-        const int h = d >> 7;                           // half: k 32h .. 32h+31 of the stage
+        // tcgen05.st reaches only the warp's TMEM lane quarter (warp % 4), so the
+        // weight row of a thread is its TMEM lane: row = 32 * (warp % 4) + lane.
+        const int dw = warp - kDec0;                    // 0 .. kDecodeWarps-1
+        const int d = dw * 32 + lane;                   // code-ring slot, 0 .. kDecodeThreads-1
+        const int r = (warp & 3) * 32 + lane;           // weight row within the tile
+        const int h = dw >> 2;                          // half: k 32h .. 32h+31 of the stage
+        const uint32_t tw = tmem_base + ((uint32_t)((warp & 3) * 32) << 16) + kWCol0 + (uint32_t)(16 * h);
         const uint32_t lane4 = 4u * (uint32_t)lane;
         const int hbytes = (p.bits == 4) ? 16 : 12;     // codes of one half row per stage
         int stage = 0;
@@ -589,13 +634,11 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
                 ok = false;
                 return;
             }
-            const uint32_t wrow = ws0 + stage * kWStageBytes + r * 128;
-            const uint32_t sw = (uint32_t)(r & 7);
-#pragma unroll
-            for (int i = 0; i < 4; ++i)
-                sts128(wrow + ((((uint32_t)(4 * h + i)) ^ sw) << 4), cur_pr[4 * i], cur_pr[4 * i + 1],
-                       cur_pr[4 * i + 2], cur_pr[4 * i + 3]);
-            fence_proxy_async();          // this thread's tile writes -> visible to the tensor core
+            tc_fence_after();
+            // pair q holds k = 32h + 2q (low half) and 32h + 2q + 1: column 16h + q of the stage
+            tmem_st16(tw + (uint32_t)stage * kWStageCols, cur_pr);
+            tmem_wait_st();
+            tc_fence_before();            // this warp's tensor-memory writes -> the MMA issuer
             __syncwarp();
             if (lane == 0) mbar_arrive(wfull(stage));
             if (++stage == kWStages) { stage = 0; phase ^= 1u; }
@@ -652,8 +695,8 @@ uint32_t make_idesc(bool f16_inputs)
     return d;
 }
 
-// Dynamic shared memory of the layout: table rows, X and W stages, barriers.
-constexpr uint32_t kSmemBytes = kTabRegion + kXStages * kXStageBytes + kWStages * kWStageBytes + 256;
+// Dynamic shared memory of the layout: table rows, X stages, barriers.
+constexpr uint32_t kSmemBytes = kTabRegion + kXStages * kXStageBytes + 256;
 
 }  // namespace
 
