@@ -13,6 +13,8 @@
  * path as device kernels behind plain C calls:
  *   logq_build_codebook  host: (bits, base, range) -> levels and boundaries
  *   logq_quantize        device: fp32 W[N][K] -> packed codes + codebook
+ *   logq_quantize_energy device: the same with w_min / w_max / b derived from W
+ *                        (Sec. 3.2, Eqs. (3)-(5))
  *   logq_linear          device: codes, codebook, X[B][K] -> Y[B][N] = X * What^T
  *
  * Conventions shared by every call:
@@ -181,6 +183,41 @@ logq_status logq_linear(const uint8_t* codes, const logq_codebook* cb, const voi
 logq_status logq_quantize_noalloc(const float* W, int64_t N, int64_t K, int bits, double base,
                                   double range, int flags, uint8_t* codes,
                                   logq_codebook* cb_out, void* stream);
+
+/* Bytes of device scratch that logq_quantize_energy needs (a constant, about
+ * 65 KB).  Caller-allocated, 16-byte aligned; its contents need no
+ * initialisation and are overwritten by every call. */
+size_t logq_energy_scratch_bytes(void);
+
+/*
+ * Self-calibrating quantisation (Sec. 3.2): derive the effective range of
+ * W[N][K] (device, fp32) from the weights and quantise with it.
+ *   w_max = max_i |w_i|;
+ *   w_min = min { t : sum_{|w_i| <= t} w_i^2 / sum_i w_i^2 >= eps }   (Eq. (5)),
+ *           the smallest weight magnitude at which the discarded energy share
+ *           reaches eps (the paper uses eps = 4e-3 at 4 bits); it is always
+ *           one of the |w_i|;
+ *   b     = (w_max / w_min)^(1 / q_max)                                (Eq. (3));
+ *   then the codebook (bits, b, w_max, flags) -- flags LOGQ_SHIFT_FLOOR is
+ *   Eq. (4) as printed -- and the codes exactly as logq_quantize with those
+ *   arguments would produce them.
+ * The selection runs on the device in three streaming passes over W (a radix
+ * selection over the bit patterns of |w|) plus the quantisation pass; energies of equal-exponent buckets are summed exactly in
+ * integers and accumulated across buckets in fp64, in ascending order of |w|.
+ *   eps in (0, 1].  wmin_out (host, may be NULL) receives w_min; cb_out (host,
+ *   may be NULL) the codebook (its base is b, its range w_max).
+ *   scratch: logq_energy_scratch_bytes() bytes of device memory.
+ * Synchronises `stream` once after the range is known and once before
+ * returning.
+ * Errors: those of logq_quantize; LOGQ_ERR_INVALID_ARG also when eps is not in
+ * (0, 1], W is all zero, or w_min == w_max (a single magnitude holds the
+ * required energy, so Eq. (3) gives b = 1: no logarithmic codebook exists);
+ * LOGQ_ERR_WORKSPACE also for a missing, small or misaligned scratch.
+ */
+logq_status logq_quantize_energy(const float* W, int64_t N, int64_t K, int bits, double eps, int flags,
+                                 uint8_t* codes, logq_codebook* cb_out, double* wmin_out,
+                                 void* workspace, size_t workspace_bytes, void* scratch,
+                                 size_t scratch_bytes, void* stream);
 
 /* One matrix of logq_linear_grouped. */
 typedef struct logq_linear_item {

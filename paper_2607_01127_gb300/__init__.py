@@ -38,7 +38,8 @@ LOGQ_SHIFT_EXACT, LOGQ_SHIFT_FLOOR = 0, 1
 
 EXPORTED = ("logq_build_codebook", "logq_packed_bytes", "logq_workspace_bytes", "logq_quantize",
             "logq_linear", "logq_workspace_status", "logq_status_string", "logq_device_sm_count",
-            "logq_quantize_noalloc", "logq_linear_grouped")
+            "logq_quantize_noalloc", "logq_linear_grouped", "logq_energy_scratch_bytes",
+            "logq_quantize_energy")
 
 
 class Codebook(ctypes.Structure):
@@ -91,6 +92,11 @@ def _load() -> ctypes.CDLL:
     lib.logq_quantize_noalloc.argtypes = [P, c_i64, c_i64, c_int, c_dbl, c_dbl, c_int, P,
                                           ctypes.POINTER(Codebook), P]
     lib.logq_quantize_noalloc.restype = c_int
+    lib.logq_energy_scratch_bytes.argtypes = []
+    lib.logq_energy_scratch_bytes.restype = ctypes.c_size_t
+    lib.logq_quantize_energy.argtypes = [P, c_i64, c_i64, c_int, c_dbl, c_int, P, ctypes.POINTER(Codebook),
+                                         ctypes.POINTER(c_dbl), P, ctypes.c_size_t, P, ctypes.c_size_t, P]
+    lib.logq_quantize_energy.restype = c_int
     lib.logq_linear.argtypes = [P, ctypes.POINTER(Codebook), P, c_int, c_i64, c_i64, c_i64, P,
                                 c_int, P, ctypes.c_size_t, P]
     lib.logq_linear.restype = c_int
@@ -206,6 +212,34 @@ def logq_quantize_noalloc(W, bits: int, base: float, range_: float = 0.0,
                                       ctypes.byref(cb), _stream_ptr(stream))
     _check(st, "logq_quantize_noalloc")
     return codes[:nbytes], cb
+
+
+def logq_energy_scratch_bytes() -> int:
+    return int(_lib().logq_energy_scratch_bytes())
+
+
+def logq_quantize_energy(W, bits: int, eps: float = 4e-3, flags: int = LOGQ_SHIFT_EXACT, codes=None,
+                         workspace=None, scratch=None, stream=None):
+    """Self-calibrating quantisation (Sec. 3.2, Eqs. (3)-(5)): w_max = max|W|, w_min from the
+    energy share eps, b = (w_max / w_min)^(1 / q_max).  Returns (codes, Codebook, w_min)."""
+    import torch
+    assert W.dtype == torch.float32 and W.is_cuda and W.dim() == 2 and W.is_contiguous()
+    N, K = W.shape
+    nbytes = logq_packed_bytes(N, K, bits)
+    if codes is None:
+        codes = torch.empty(max(nbytes, 16), dtype=torch.uint8, device=W.device)
+    if workspace is None:
+        workspace = new_workspace(W.device)
+    if scratch is None:
+        scratch = torch.empty(logq_energy_scratch_bytes(), dtype=torch.uint8, device=W.device)
+    cb = Codebook()
+    wmin = ctypes.c_double(0.0)
+    st = _lib().logq_quantize_energy(ctypes.c_void_p(W.data_ptr()), N, K, int(bits), float(eps), int(flags),
+                                     ctypes.c_void_p(codes.data_ptr()), ctypes.byref(cb), ctypes.byref(wmin),
+                                     ctypes.c_void_p(workspace.data_ptr()), workspace.numel(),
+                                     ctypes.c_void_p(scratch.data_ptr()), scratch.numel(), _stream_ptr(stream))
+    _check(st, "logq_quantize_energy")
+    return codes[:nbytes], cb, wmin.value
 
 
 def logq_linear(codes, cb: Codebook, X, N: int, K: int, y_dtype=None, Y=None, workspace=None,

@@ -19,6 +19,21 @@ struct Workspace {
 static_assert(sizeof(Workspace) == 256, "workspace layout");
 constexpr size_t kWorkspaceBytes = sizeof(Workspace);
 
+// Device state of the energy-range selection (caller-provided scratch,
+// logq_energy_scratch_bytes() bytes): bucket energies of the current level as
+// exact integer sums of the high / low 24 bits of m^2, the total energy, the
+// energy below the selected prefix, the prefix and the result.
+struct EnergyState {
+    unsigned long long hi[4096];
+    unsigned long long lo[4096];
+    double total;
+    double below;
+    uint32_t prefix;
+    uint32_t wmin_bits;
+    uint32_t failed;        // the window pass found the crossing below its window
+    uint32_t _pad;
+};
+
 // Decision boundaries handed to the quantise kernel (fp32, rounded up).
 struct QuantParams {
     float thresh[8];
@@ -65,6 +80,8 @@ struct GroupArgs {
 
 int sm_count();
 cudaError_t launch_absmax(const float* W, int64_t count, Workspace* ws, cudaStream_t s);
+cudaError_t launch_energy_range(const float* W, int64_t count, double eps, EnergyState* st, Workspace* ws,
+                                cudaStream_t s);
 cudaError_t launch_quantize(const float* W, int64_t N, int64_t K, const QuantParams& p,
                             uint8_t* codes, Workspace* ws, cudaStream_t s);
 cudaError_t launch_gemv(const LinearArgs& a, cudaStream_t s);

@@ -196,6 +196,61 @@ logq_status logq_quantize(const float* W, int64_t N, int64_t K, int bits, double
     return LOGQ_OK;
 }
 
+size_t logq_energy_scratch_bytes(void) { return sizeof(EnergyState); }
+
+logq_status logq_quantize_energy(const float* W, int64_t N, int64_t K, int bits, double eps, int flags,
+                                 uint8_t* codes, logq_codebook* cb_out, double* wmin_out,
+                                 void* workspace, size_t workspace_bytes, void* scratch,
+                                 size_t scratch_bytes, void* stream)
+{
+    if (!W || !codes || !aligned16(W) || !aligned16(codes)) return LOGQ_ERR_INVALID_ARG;
+    if (logq_packed_bytes(N, K, bits) == 0) return LOGQ_ERR_INVALID_ARG;
+    if (!isfinite(eps) || !(eps > 0.0) || eps > 1.0) return LOGQ_ERR_INVALID_ARG;
+    if (flags != LOGQ_SHIFT_EXACT && flags != LOGQ_SHIFT_FLOOR) return LOGQ_ERR_INVALID_ARG;
+    if (!workspace || !aligned16(workspace) || workspace_bytes < kWorkspaceBytes) return LOGQ_ERR_WORKSPACE;
+    if (!scratch || !aligned16(scratch) || scratch_bytes < sizeof(EnergyState)) return LOGQ_ERR_WORKSPACE;
+    if (N > (int64_t(1) << 40) / K) return LOGQ_ERR_INVALID_ARG;
+
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    Workspace* ws = static_cast<Workspace*>(workspace);
+    EnergyState* st = static_cast<EnergyState*>(scratch);
+    cudaError_t e = cudaMemsetAsync(ws, 0, 2 * sizeof(uint32_t), s);
+    if (e != cudaSuccess) return LOGQ_ERR_CUDA;
+    // Sec. 3.2: w_max and the Eq. (5) w_min, on the device
+    if ((e = launch_energy_range(W, N * K, eps, st, ws, s)) != cudaSuccess) return LOGQ_ERR_CUDA;
+    uint32_t host_words[2] = {0, 0}, sel[2] = {0, 0};      // sel: w_min bits, window failure
+    if ((e = cudaMemcpyAsync(host_words, ws, sizeof host_words, cudaMemcpyDeviceToHost, s)) != cudaSuccess)
+        return LOGQ_ERR_CUDA;
+    if ((e = cudaMemcpyAsync(sel, &st->wmin_bits, sizeof sel, cudaMemcpyDeviceToHost, s)) != cudaSuccess)
+        return LOGQ_ERR_CUDA;
+    if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return LOGQ_ERR_CUDA;
+    if (host_words[1]) return LOGQ_ERR_NONFINITE;
+    float fmax, fmin;
+    memcpy(&fmax, &host_words[0], 4);
+    memcpy(&fmin, &sel[0], 4);
+    if (!(fmax > 0.0f)) return LOGQ_ERR_INVALID_ARG;     // all-zero weights
+    if (sel[1]) return LOGQ_ERR_CUDA;                    // selection inconsistent (not expected)
+    if (!(fmin > 0.0f)) return LOGQ_ERR_INVALID_ARG;
+    if (!(fmin < fmax)) return LOGQ_ERR_INVALID_ARG;                      // Eq. (3) would give b = 1
+    const int qmax = (1 << (bits - 1)) - 1;
+    const double base = pow((double)fmax / (double)fmin, 1.0 / (double)qmax);   // Eq. (3)
+
+    logq_codebook cb;
+    logq_status st_cb = logq_build_codebook(bits, base, (double)fmax, flags, &cb);
+    if (st_cb != LOGQ_OK) return st_cb;
+    QuantParams p;
+    memset(&p, 0, sizeof p);
+    for (int j = 0; j < 8; ++j) p.thresh[j] = cb.thresh[j];
+    p.qmax = cb.qmax;
+    p.bits = bits;
+    p.check_nonfinite = 0;          // the range pass already looked at every weight
+    if ((e = launch_quantize(W, N, K, p, codes, ws, s)) != cudaSuccess) return LOGQ_ERR_CUDA;
+    if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return LOGQ_ERR_CUDA;
+    if (cb_out) *cb_out = cb;
+    if (wmin_out) *wmin_out = (double)fmin;
+    return LOGQ_OK;
+}
+
 logq_status logq_linear(const uint8_t* codes, const logq_codebook* cb, const void* X,
                         logq_dtype x_dtype, int64_t B, int64_t N, int64_t K, void* Y,
                         logq_dtype y_dtype, void* workspace, size_t workspace_bytes, void* stream)

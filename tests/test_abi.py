@@ -133,6 +133,33 @@ def test_quantize_rejects_before_launch(logq):
     assert call(ws=_fake(0x30008)) == logq.LOGQ_ERR_WORKSPACE
 
 
+def test_energy_quantize_rejects_before_launch(logq):
+    """logq_quantize_energy validates eps, sizes, workspace and scratch on the
+    host before anything is enqueued (fake device addresses, no GPU)."""
+    L = logq.lib
+    W, C, ws, sc = _fake(0x10000), _fake(0x20000), _fake(0x30000), _fake(0x40000)
+    cb = logq.Codebook()
+    wmin = ctypes.c_double(0.0)
+    scb = L.logq_energy_scratch_bytes()
+    assert 16 * 1024 < scb < 128 * 1024
+
+    def call(W=W, C=C, ws=ws, wsb=256, sc=sc, scb=scb, N=4, K=128, bits=4, eps=4e-3, flags=0):
+        return L.logq_quantize_energy(W, N, K, bits, eps, flags, C, ctypes.byref(cb), ctypes.byref(wmin),
+                                      ws, wsb, sc, scb, None)
+
+    assert call(W=None) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(C=_fake(0x20008)) == logq.LOGQ_ERR_INVALID_ARG         # misaligned
+    assert call(K=100) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(bits=2) == logq.LOGQ_ERR_INVALID_ARG
+    for eps in (0.0, -1e-3, 1.0000001, float("nan"), float("inf")):
+        assert call(eps=eps) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(flags=3) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(ws=None) == logq.LOGQ_ERR_WORKSPACE
+    assert call(sc=None) == logq.LOGQ_ERR_WORKSPACE
+    assert call(scb=scb - 8) == logq.LOGQ_ERR_WORKSPACE
+    assert call(sc=_fake(0x40004)) == logq.LOGQ_ERR_WORKSPACE
+
+
 def test_linear_rejects_before_launch(logq):
     L = logq.lib
     cb = logq.logq_build_codebook(4, 1.5, 1.0)
