@@ -52,12 +52,12 @@ class Codebook(ctypes.Structure):
         ("base", ctypes.c_double),
         ("range", ctypes.c_double),
         ("shift", ctypes.c_double),
-        ("level", ctypes.c_double * 8),
-        ("tau", ctypes.c_double * 8),
-        ("level32", ctypes.c_float * 8),
-        ("tau32_up", ctypes.c_float * 8),
-        ("level_bf16", ctypes.c_uint16 * 8),
-        ("level_f16", ctypes.c_uint16 * 8),
+        ("level", ctypes.c_double * 128),
+        ("tau", ctypes.c_double * 128),
+        ("level32", ctypes.c_float * 128),
+        ("tau32_up", ctypes.c_float * 128),
+        ("level_bf16", ctypes.c_uint16 * 128),
+        ("level_f16", ctypes.c_uint16 * 128),
     ]
 
     @property

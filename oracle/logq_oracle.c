@@ -43,6 +43,7 @@
  *          f_p = code(2p) | code(2p+1) << 3.  For p = 5i + j (i < 3, j < 5)
  *          f_p sits in bits [6j, 6j+6) of W_i; f_15 is split two bits per
  *          word: bits 30-31 of W0, W1, W2 hold f_15 bits 0-1, 2-3, 4-5.
+ *   n = 8: row-major [N][K] bytes, one code per byte (sign in bit 7).
  */
 #include <math.h>
 #include <stdint.h>
@@ -63,12 +64,12 @@ typedef struct {
     double base;           /* b */
     double range;          /* w_max handed in */
     double shift;          /* s */
-    double level[8];       /* L_m = b^(m - s), m = 0..q_max, L_0 = 0 (Eq. (2)) */
-    double tau[8];         /* tau_j = b^(j + 1/2 - s), j = 0..q_max-1 (R3) */
-    float level32[8];      /* L_m rounded to nearest-even fp32 */
-    float tau32_up[8];     /* smallest fp32 >= tau_j */
-    uint16_t level_bf16[8];/* level32 rounded to nearest-even bf16 (bits) */
-    uint16_t level_f16[8]; /* level32 rounded to nearest-even fp16 (bits) */
+    double level[128];     /* L_m = b^(m - s), m = 0..q_max, L_0 = 0 (Eq. (2)) */
+    double tau[128];       /* tau_j = b^(j + 1/2 - s), j = 0..q_max-1 (R3) */
+    float level32[128];    /* L_m rounded to nearest-even fp32 */
+    float tau32_up[128];   /* smallest fp32 >= tau_j */
+    uint16_t level_bf16[128];/* level32 rounded to nearest-even bf16 (bits) */
+    uint16_t level_f16[128]; /* level32 rounded to nearest-even fp16 (bits) */
 } oracle_codebook;
 
 /* ------------------------------------------------------------------ */
@@ -153,7 +154,7 @@ static long floor_log_b(double x, double b)
 int oracle_build_codebook(int bits, double base, double range, int shift_mode,
                           oracle_codebook* cb)
 {
-    if (bits < 2 || bits > 8 || !(base > 1.0) || !isfinite(base) ||
+    if ((bits != 3 && bits != 4 && bits != 8) || !(base > 1.0) || !isfinite(base) ||
         !(range > 0.0) || !isfinite(range))
         return 1;
     memset(cb, 0, sizeof *cb);
@@ -162,7 +163,6 @@ int oracle_build_codebook(int bits, double base, double range, int shift_mode,
     cb->shift_mode = shift_mode;
     cb->base = base;
     cb->range = range;
-    if (cb->qmax > 7) return 1;            /* tables here hold up to 8 levels */
     double lb_range = log(range) / log(base);
     if (shift_mode == ORACLE_SHIFT_FLOOR)
         cb->shift = (double)cb->qmax - (double)floor_log_b(range, base);
@@ -272,6 +272,7 @@ static int8_t value_of(unsigned code, int bits)
 
 int64_t oracle_packed_row_bytes(int64_t K, int bits)
 {
+    if (bits == 8) return K;
     if (bits == 4) return K / 2;
     if (bits == 3) return (K / 32) * 12;
     return -1;
@@ -285,7 +286,9 @@ int oracle_pack(const int8_t* q, int64_t N, int64_t K, int bits, uint8_t* out)
     for (int64_t r = 0; r < N; ++r) {
         const int8_t* qr = q + r * K;
         uint8_t* o = out + r * rb;
-        if (bits == 4) {
+        if (bits == 8) {
+            for (int64_t k = 0; k < K; ++k) o[k] = (uint8_t)code_of(qr[k], 8);
+        } else if (bits == 4) {
             for (int64_t j = 0; j < K / 2; ++j)
                 o[j] = (uint8_t)(code_of(qr[2 * j], 4) | (code_of(qr[2 * j + 1], 4) << 4));
         } else {
@@ -320,7 +323,9 @@ int oracle_unpack(const uint8_t* packed, int64_t N, int64_t K, int bits, int8_t*
     for (int64_t r = 0; r < N; ++r) {
         const uint8_t* p = packed + r * rb;
         int8_t* qr = q + r * K;
-        if (bits == 4) {
+        if (bits == 8) {
+            for (int64_t k = 0; k < K; ++k) qr[k] = value_of(p[k], 8);
+        } else if (bits == 4) {
             for (int64_t j = 0; j < K / 2; ++j) {
                 qr[2 * j] = value_of(p[j] & 0xFu, 4);
                 qr[2 * j + 1] = value_of(p[j] >> 4, 4);
