@@ -84,17 +84,17 @@ typedef enum {
  *   (bit patterns); logq_linear multiplies with the table of X's dtype.
  */
 typedef struct logq_codebook {
-    int32_t bits;            /* n: 3 or 4 */
+    int32_t bits;            /* n: 3, 4 or 8 */
     int32_t qmax;            /* 2^(n-1) - 1 */
     int32_t flags;           /* LOGQ_SHIFT_* used */
     int32_t _pad;
     double base;             /* b */
     double shift;            /* s */
     double range;            /* w_max the codebook was built for */
-    float level[16];
-    float thresh[8];
-    uint16_t level_bf16[16];
-    uint16_t level_f16[16];
+    float level[256];        /* entries 0 .. 2^n - 1 used */
+    float thresh[128];       /* entries 0 .. q_max - 1 used */
+    uint16_t level_bf16[256];
+    uint16_t level_f16[256];
 } logq_codebook;
 
 /*
@@ -103,6 +103,7 @@ typedef struct logq_codebook {
  *   only for negative weights with m > 0.
  *   n = 4: [N][K/2] bytes; byte j of a row holds k = 2j in bits 0-3 and
  *          k = 2j+1 in bits 4-7.
+ *   n = 8: [N][K] bytes, one code per byte (sign in bit 7).
  *   n = 3: [N][3K/8] bytes; each run of 32 k is a 12-byte group of three
  *          little-endian uint32 W0, W1, W2.  Pair p (k = 2p, 2p+1 of the group)
  *          is the 6-bit field f_p = c(2p) | c(2p+1) << 3; for p = 5i + j
@@ -113,13 +114,13 @@ typedef struct logq_codebook {
 
 /* Fill *out for an n-bit codebook with base b = base > 1 and range > 0
  * (Eq. (2) levels, Eq. (4) shift per flags).  Host only, no CUDA call.
- * Errors: LOGQ_ERR_INVALID_ARG for bits not in {3,4}, base <= 1 or not
+ * Errors: LOGQ_ERR_INVALID_ARG for bits not in {3,4,8}, base <= 1 or not
  * finite, range <= 0 or not finite, unknown flags, out == NULL. */
 logq_status logq_build_codebook(int bits, double base, double range, int flags,
                                 logq_codebook* out);
 
-/* Bytes of packed codes for an N x K matrix at n bits (N*K/2 or N*3K/8);
- * 0 when N <= 0, K is not a positive multiple of 128 or bits not in {3,4}. */
+/* Bytes of packed codes for an N x K matrix at n bits (N*K/2, N*3K/8 or N*K);
+ * 0 when N <= 0, K is not a positive multiple of 128 or bits not in {3,4,8}. */
 size_t logq_packed_bytes(int64_t N, int64_t K, int bits);
 
 /* Bytes of device workspace that logq_quantize and logq_linear need (a small
@@ -152,8 +153,10 @@ logq_status logq_quantize(const float* W, int64_t N, int64_t K, int bits, double
  *   codes (device): packed as above for cb->bits.  X (device): x_dtype.
  *   Y (device): y_dtype in {LOGQ_F32, x_dtype}; a 16-bit Y is the fp32 sum
  *   rounded to nearest-even.  All device pointers 16-byte aligned.
- *   B <= 16 runs the decode GEMV / skinny-GEMM kernel on CUDA cores;
- *   B > 16 runs the prefill GEMM kernel on the tensor cores (tcgen05).
+ *   B <= 16 (4-bit) or B <= 4 (3- and 8-bit) runs the decode GEMV /
+ *   skinny-GEMM kernel on CUDA cores; larger B runs the prefill GEMM kernel
+ *   on the tensor cores (tcgen05) for 3- and 4-bit codes and returns
+ *   LOGQ_ERR_UNSUPPORTED for 8-bit codes.
  * Asynchronous.  Errors: LOGQ_ERR_INVALID_ARG, LOGQ_ERR_UNSUPPORTED,
  * LOGQ_ERR_WORKSPACE, LOGQ_ERR_CUDA (launch).  A device-side wait that hit
  * its bound is reported later by logq_workspace_status. */
@@ -232,7 +235,7 @@ typedef struct logq_linear_item {
  * e.g. the q/k/v or the gate/up projections of a transformer layer -- each
  * with its own per-tensor codebook (Sec. 3.1) and output: Y_i = X * What_i^T
  * (Sec. 3.3), in one call.  count is 1..4 and all items share the code width
- * of their codebooks.  With B <= 16 (4-bit) or B <= 4 (3-bit) the matrices
+ * of their codebooks.  With B <= 16 (4-bit) or B <= 4 (3-, 8-bit) the matrices
  * share a single decode-GEMV launch; larger B runs one prefill launch each.
  * l2_prefetch (device, may be NULL) / l2_prefetch_bytes name a range the
  * call asks the L2 cache to fetch while it runs -- for a decode step, the

@@ -52,10 +52,10 @@ class Codebook(ctypes.Structure):
         ("base", ctypes.c_double),
         ("shift", ctypes.c_double),
         ("range", ctypes.c_double),
-        ("level", ctypes.c_float * 16),
-        ("thresh", ctypes.c_float * 8),
-        ("level_bf16", ctypes.c_uint16 * 16),
-        ("level_f16", ctypes.c_uint16 * 16),
+        ("level", ctypes.c_float * 256),
+        ("thresh", ctypes.c_float * 128),
+        ("level_bf16", ctypes.c_uint16 * 256),
+        ("level_f16", ctypes.c_uint16 * 256),
     ]
 
 

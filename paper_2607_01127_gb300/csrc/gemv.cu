@@ -31,6 +31,8 @@
 #include <stdint.h>
 #include <string.h>
 
+#include <type_traits>
+
 #include "internal.h"
 
 namespace logq {
@@ -108,6 +110,18 @@ struct GemvParams {
     int64_t pf_share;     // bytes of that range per CTA (multiple of 16)
 };
 
+// 8-bit codes: their 256 code-indexed levels per matrix travel as a second
+// kernel parameter of the 8-bit kernels only, so the 3- and 4-bit launches keep
+// their small parameter block.
+struct Levels8 {
+    uint16_t v[kMaxItems][256];
+};
+struct NoLevels {
+    int32_t unused;
+};
+template <int BITS>
+using LevelsT = typename std::conditional<BITS == 8, Levels8, NoLevels>::type;
+
 __device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel)
 {
     uint32_t r;
@@ -161,6 +175,30 @@ __device__ __forceinline__ void fma_pair(float& a0, float& a1, uint32_t w, uint3
             "fma.rn.f32.bf16 %0, wl, xl, %0;\n\t"
             "fma.rn.f32.bf16 %1, wh, xh, %1;}"
             : "+f"(a0), "+f"(a1) : "r"(w), "r"(x));
+    }
+}
+
+// 8-bit: two looked-up entries (each holding its 16-bit value in both halves)
+// times one activation pair.
+template <bool F16>
+__device__ __forceinline__ void fma_two(float& a0, float& a1, uint32_t w0, uint32_t w1, uint32_t x)
+{
+    if constexpr (F16) {
+        asm("{.reg .b16 al, ah, bl, bh, xl, xh;\n\t"
+            "mov.b32 {al, ah}, %2;\n\t"
+            "mov.b32 {bl, bh}, %3;\n\t"
+            "mov.b32 {xl, xh}, %4;\n\t"
+            "fma.rn.f32.f16 %0, al, xl, %0;\n\t"
+            "fma.rn.f32.f16 %1, bl, xh, %1;}"
+            : "+f"(a0), "+f"(a1) : "r"(w0), "r"(w1), "r"(x));
+    } else {
+        asm("{.reg .b16 al, ah, bl, bh, xl, xh;\n\t"
+            "mov.b32 {al, ah}, %2;\n\t"
+            "mov.b32 {bl, bh}, %3;\n\t"
+            "mov.b32 {xl, xh}, %4;\n\t"
+            "fma.rn.f32.bf16 %0, al, xl, %0;\n\t"
+            "fma.rn.f32.bf16 %1, bl, xh, %1;}"
+            : "+f"(a0), "+f"(a1) : "r"(w0), "r"(w1), "r"(x));
     }
 }
 
@@ -232,7 +270,20 @@ template <int BITS, int B, int NW, bool F16, int NPAIR>
 __device__ __forceinline__ void decode_row(const CodeVec<NW>& c, uint32_t base_lane,
                                            const uint32_t (&xr)[B][NPAIR], float* acc, float* acc_hi)
 {
-    if constexpr (BITS == 4) {
+    if constexpr (BITS == 8) {
+        // word wi holds the codes of k = 4 wi .. 4 wi + 3, one per byte
+#pragma unroll
+        for (int wi = 0; wi < NW; ++wi) {
+            uint32_t o[4];
+            addrs4(c.w[wi], base_lane, o);
+            const uint32_t v0 = lds_tab(o[0]), v1 = lds_tab(o[1]), v2 = lds_tab(o[2]), v3 = lds_tab(o[3]);
+#pragma unroll
+            for (int b = 0; b < B; ++b) {
+                fma_two<F16>(acc[b], acc_hi[b], v0, v1, xr[b][2 * wi]);
+                fma_two<F16>(acc[b], acc_hi[b], v2, v3, xr[b][2 * wi + 1]);
+            }
+        }
+    } else if constexpr (BITS == 4) {
 #pragma unroll
         for (int wi = 0; wi < NW; ++wi) {
             uint32_t o[4];
@@ -261,12 +312,13 @@ __device__ __forceinline__ void decode_row(const CodeVec<NW>& c, uint32_t base_l
 }
 
 template <int BITS, int B, int KW, int R, bool F16, int NT>
-__global__ void __launch_bounds__(NT, 512 / NT) gemv_kernel(const __grid_constant__ GemvParams p)
+__global__ void __launch_bounds__(NT, 512 / NT) gemv_kernel(const __grid_constant__ GemvParams p,
+                                                            const __grid_constant__ LevelsT<BITS> lv)
 {
     extern __shared__ __align__(16) uint8_t smem[];
     constexpr int NPAIR = KW / 2;                            // bf16 pairs of x per lane and batch row
-    constexpr int NW = (BITS == 4) ? KW / 8 : 3 * KW / 32;   // code words per lane and row
-    constexpr int NENT = (BITS == 4) ? 256 : 64;
+    constexpr int NW = (BITS == 8) ? KW / 4 : (BITS == 4) ? KW / 8 : 3 * KW / 32;   // code words per lane and row
+    constexpr int NENT = (BITS == 3) ? 64 : 256;
     constexpr uint32_t TAB_BYTES = NENT * kTabStride;
     constexpr int V = R * B;
     constexpr int SPAN = 32 * KW;
@@ -304,7 +356,8 @@ __global__ void __launch_bounds__(NT, 512 / NT) gemv_kernel(const __grid_constan
         k0 = s * SPAN + lane * KW;
         active = k0 < p.K;
         // idle lanes read the row start (valid memory) and multiply by zero
-        const int64_t lane_byte = active ? ((BITS == 4) ? (int64_t)k0 / 2 : (int64_t)k0 / 32 * 12) : 0;
+        const int64_t lane_byte =
+            active ? ((BITS == 8) ? (int64_t)k0 : (BITS == 4) ? (int64_t)k0 / 2 : (int64_t)k0 / 32 * 12) : 0;
         return item.codes + (q0 + g) * p.row_bytes + lane_byte;
     };
     // codes of the round whose first row is at rp, here = rows left from it
@@ -357,15 +410,24 @@ __global__ void __launch_bounds__(NT, 512 / NT) gemv_kernel(const __grid_constan
     //    code) << 16, 32 copies (one per lane) in the first 128 bytes of its
     //    256-byte row.  The 16 levels are staged in the free half of row 0
     //    (indexed parameter reads with per-thread indices would serialise).
-    uint32_t* lvl = reinterpret_cast<uint32_t*>(smem + kLvlOff);
-    if (tid < 16) lvl[tid] = item.lvl16[tid] & 0xffffu;
-    __syncthreads();
-    for (int i = tid; i < NENT * 8; i += NT) {
-        const int e = i >> 3, part = i & 7;
-        const uint32_t lo = (BITS == 4) ? (e & 15) : (e & 7);
-        const uint32_t hi = (BITS == 4) ? (e >> 4) : (e >> 3);
-        const uint32_t v = lvl[lo] | (lvl[hi] << 16);
-        reinterpret_cast<uint4*>(smem + e * kTabStride)[part] = make_uint4(v, v, v, v);
+    //    8-bit codes: entry e is the value of code e in both halves.
+    if constexpr (BITS == 8) {
+        for (int i = tid; i < NENT * 8; i += NT) {
+            const int e = i >> 3, part = i & 7;
+            const uint32_t v = (uint32_t)lv.v[m][e] * 0x10001u;
+            reinterpret_cast<uint4*>(smem + e * kTabStride)[part] = make_uint4(v, v, v, v);
+        }
+    } else {
+        uint32_t* lvl = reinterpret_cast<uint32_t*>(smem + kLvlOff);
+        if (tid < 16) lvl[tid] = item.lvl16[tid] & 0xffffu;
+        __syncthreads();
+        for (int i = tid; i < NENT * 8; i += NT) {
+            const int e = i >> 3, part = i & 7;
+            const uint32_t lo = (BITS == 4) ? (e & 15) : (e & 7);
+            const uint32_t hi = (BITS == 4) ? (e >> 4) : (e >> 3);
+            const uint32_t v = lvl[lo] | (lvl[hi] << 16);
+            reinterpret_cast<uint4*>(smem + e * kTabStride)[part] = make_uint4(v, v, v, v);
+        }
     }
     // span partial i (in the free half of table row i / 32, or after the table)
     auto red = [&](int i) -> float& {
@@ -506,8 +568,13 @@ struct Config {
 // Dynamic shared memory opt-in and a carveout that leaves room for two CTAs
 // per SM: per-device function attributes, set once per device.
 template <int BITS, int B, int KW, int R, bool F16, int NT>
-cudaError_t run(const GemvParams& p, int grid, size_t smem, cudaStream_t s)
+cudaError_t run(const GemvParams& p, const GroupArgs& a, int grid, size_t smem, cudaStream_t s)
 {
+    LevelsT<BITS> lv;
+    memset(&lv, 0, sizeof lv);
+    if constexpr (BITS == 8)
+        for (int i = 0; i < a.count; ++i)
+            for (int c = 0; c < 256; ++c) lv.v[i][c] = a.item[i].lvl16[c];
     auto k = gemv_kernel<BITS, B, KW, R, F16, NT>;
     static bool configured[64] = {false};
     int dev = 0;
@@ -532,29 +599,35 @@ cudaError_t run(const GemvParams& p, int grid, size_t smem, cudaStream_t s)
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, k, p);
+    return cudaLaunchKernelEx(&cfg, k, p, lv);
 }
 
 template <bool F16>
-cudaError_t dispatch(int bits, int Bp, bool large, bool tiny, const GemvParams& p, int grid, size_t smem,
-                     cudaStream_t s)
+cudaError_t dispatch(int bits, int Bp, bool large, bool tiny, const GemvParams& p, const GroupArgs& a, int grid,
+                     size_t smem, cudaStream_t s)
 {
     constexpr int L = kLargeThreads, S = kSmallThreads;
-    if (bits == 4) {
+    if (bits == 8) {
+        switch (Bp) {
+        case 1: return large ? run<8, 1, 16, 8, F16, L>(p, a, grid, smem, s) : run<8, 1, 16, 8, F16, S>(p, a, grid, smem, s);
+        case 2: return large ? run<8, 2, 16, 4, F16, L>(p, a, grid, smem, s) : run<8, 2, 16, 4, F16, S>(p, a, grid, smem, s);
+        case 4: return run<8, 4, 16, 2, F16, S>(p, a, grid, smem, s);
+        }
+    } else if (bits == 4) {
         switch (Bp) {
         case 1:
-            if (large) return run<4, 1, 32, 8, F16, L>(p, grid, smem, s);
-            return tiny ? run<4, 1, 16, 8, F16, S>(p, grid, smem, s) : run<4, 1, 32, 8, F16, S>(p, grid, smem, s);
-        case 2: return large ? run<4, 2, 32, 4, F16, L>(p, grid, smem, s) : run<4, 2, 32, 4, F16, S>(p, grid, smem, s);
-        case 4: return run<4, 4, 16, 2, F16, S>(p, grid, smem, s);
-        case 8: return run<4, 8, 8, 1, F16, S>(p, grid, smem, s);
-        case 16: return run<4, 16, 8, 1, F16, S>(p, grid, smem, s);
+            if (large) return run<4, 1, 32, 8, F16, L>(p, a, grid, smem, s);
+            return tiny ? run<4, 1, 16, 8, F16, S>(p, a, grid, smem, s) : run<4, 1, 32, 8, F16, S>(p, a, grid, smem, s);
+        case 2: return large ? run<4, 2, 32, 4, F16, L>(p, a, grid, smem, s) : run<4, 2, 32, 4, F16, S>(p, a, grid, smem, s);
+        case 4: return run<4, 4, 16, 2, F16, S>(p, a, grid, smem, s);
+        case 8: return run<4, 8, 8, 1, F16, S>(p, a, grid, smem, s);
+        case 16: return run<4, 16, 8, 1, F16, S>(p, a, grid, smem, s);
         }
     } else {
         switch (Bp) {
-        case 1: return large ? run<3, 1, 32, 8, F16, L>(p, grid, smem, s) : run<3, 1, 32, 8, F16, S>(p, grid, smem, s);
-        case 2: return large ? run<3, 2, 32, 4, F16, L>(p, grid, smem, s) : run<3, 2, 32, 4, F16, S>(p, grid, smem, s);
-        case 4: return run<3, 4, 32, 2, F16, S>(p, grid, smem, s);
+        case 1: return large ? run<3, 1, 32, 8, F16, L>(p, a, grid, smem, s) : run<3, 1, 32, 8, F16, S>(p, a, grid, smem, s);
+        case 2: return large ? run<3, 2, 32, 4, F16, L>(p, a, grid, smem, s) : run<3, 2, 32, 4, F16, S>(p, a, grid, smem, s);
+        case 4: return run<3, 4, 32, 2, F16, S>(p, a, grid, smem, s);
         }
     }
     return cudaErrorInvalidValue;
@@ -571,6 +644,7 @@ int padded_batch(int64_t B)
 
 int kw_for(int bits, int Bp, bool tiny)
 {
+    if (bits == 8) return 16;
     if (bits == 3) return 32;
     if (Bp == 1 && tiny) return 16;
     return Bp <= 2 ? 32 : (Bp == 4 ? 16 : 8);
@@ -599,7 +673,7 @@ cudaError_t check_shared_base()
 bool gemv_supports(int bits, int64_t B)
 {
     if (bits == 4) return B >= 1 && B <= 16;
-    if (bits == 3) return B >= 1 && B <= 4;
+    if (bits == 3 || bits == 8) return B >= 1 && B <= 4;
     return false;
 }
 
@@ -611,7 +685,7 @@ cudaError_t launch_gemv_group(const GroupArgs& a, cudaStream_t s)
     const int Bp = padded_batch(a.B);
     int64_t total_rows = 0;
     for (int i = 0; i < a.count; ++i) total_rows += a.item[i].N;
-    const int64_t row_bytes = (a.bits == 4) ? a.K / 2 : a.K / 32 * 12;
+    const int64_t row_bytes = (a.bits == 8) ? a.K : (a.bits == 4) ? a.K / 2 : a.K / 32 * 12;
     const bool tiny = a.bits == 4 && Bp == 1 && total_rows * row_bytes < kTinyBytes;
     const int KW = kw_for(a.bits, Bp, tiny);
     const int span = 32 * KW;
@@ -701,10 +775,10 @@ cudaError_t launch_gemv_group(const GroupArgs& a, cudaStream_t s)
     if (chunk > max_rows) chunk = max_rows;
     if (chunk < 1) return cudaErrorInvalidValue;
     p.chunk_rows = (int32_t)chunk;
-    const size_t tab = (size_t)(a.bits == 4 ? 256 : 64) * kTabStride;
+    const size_t tab = (size_t)(a.bits == 3 ? 64 : 256) * kTabStride;
     const size_t smem = red_in_table(a.bits, Bp) ? tab : tab + (size_t)p.spans * chunk * Bp * 4;
-    return a.x_f16 ? dispatch<true>(a.bits, Bp, large, tiny, p, grid, smem, s)
-                   : dispatch<false>(a.bits, Bp, large, tiny, p, grid, smem, s);
+    return a.x_f16 ? dispatch<true>(a.bits, Bp, large, tiny, p, a, grid, smem, s)
+                   : dispatch<false>(a.bits, Bp, large, tiny, p, a, grid, smem, s);
 }
 
 cudaError_t launch_gemv(const LinearArgs& a, cudaStream_t s)
@@ -715,7 +789,7 @@ cudaError_t launch_gemv(const LinearArgs& a, cudaStream_t s)
     g.item[0].codes = a.codes;
     g.item[0].Y = a.Y;
     g.item[0].N = a.N;
-    for (int c = 0; c < 16; ++c) g.item[0].lvl16[c] = a.lvl16[c];
+    for (int c = 0; c < 256; ++c) g.item[0].lvl16[c] = a.lvl16[c];
     g.X = a.X;
     g.B = a.B;
     g.K = a.K;

@@ -36,7 +36,7 @@ struct EnergyState {
 
 // Decision boundaries handed to the quantise kernel (fp32, rounded up).
 struct QuantParams {
-    float thresh[8];
+    float thresh[128];
     int32_t qmax;
     int32_t bits;
     int32_t check_nonfinite;
@@ -52,7 +52,7 @@ struct LinearArgs {
     int bits;
     int x_f16;              // 0: bf16 activations, 1: fp16
     int y_dtype;            // logq_dtype of Y
-    uint16_t lvl16[16];     // code-indexed 16-bit levels in X's dtype
+    uint16_t lvl16[256];    // code-indexed 16-bit levels in X's dtype (2^bits used)
     Workspace* ws;
 };
 
@@ -62,7 +62,7 @@ struct GroupItem {
     const uint8_t* codes;
     void* Y;
     int64_t N;
-    uint16_t lvl16[16];
+    uint16_t lvl16[256];
 };
 
 struct GroupArgs {

@@ -81,7 +81,7 @@ extern "C" {
 
 logq_status logq_build_codebook(int bits, double base, double range, int flags, logq_codebook* out)
 {
-    if (!out || (bits != 3 && bits != 4)) return LOGQ_ERR_INVALID_ARG;
+    if (!out || (bits != 3 && bits != 4 && bits != 8)) return LOGQ_ERR_INVALID_ARG;
     if (!isfinite(base) || !(base > 1.0) || !isfinite(range) || !(range > 0.0))
         return LOGQ_ERR_INVALID_ARG;
     if (flags != LOGQ_SHIFT_EXACT && flags != LOGQ_SHIFT_FLOOR) return LOGQ_ERR_INVALID_ARG;
@@ -102,7 +102,7 @@ logq_status logq_build_codebook(int bits, double base, double range, int flags, 
                                            : (double)qmax - log(range) / log(base);
 
     // Eq. (2): L_m = b^(m - s).  Exact mode: b^(m - q_max) * range.
-    double L[8] = {0};
+    double L[128] = {0};
     for (int m = 1; m <= qmax; ++m)
         L[m] = (flags == LOGQ_SHIFT_FLOOR) ? pow(base, (double)m - cb.shift)
                                            : range * pow(base, (double)(m - qmax));
@@ -117,7 +117,7 @@ logq_status logq_build_codebook(int bits, double base, double range, int flags, 
     }
     // Decision boundary between L_j and L_{j+1}: round(log_b|w| + s) >= j + 1
     // exactly when |w| >= b^(j + 1/2 - s).
-    for (int j = 0; j < 8; ++j) {
+    for (int j = 0; j < 128; ++j) {
         if (j < qmax) {
             const double t = (flags == LOGQ_SHIFT_FLOOR)
                                  ? pow(base, (double)j + 0.5 - cb.shift)
@@ -134,6 +134,7 @@ logq_status logq_build_codebook(int bits, double base, double range, int flags, 
 size_t logq_packed_bytes(int64_t N, int64_t K, int bits)
 {
     if (N <= 0 || K <= 0 || (K % 128) != 0) return 0;
+    if (bits == 8) return (size_t)N * (size_t)K;
     if (bits == 4) return (size_t)N * (size_t)(K / 2);
     if (bits == 3) return (size_t)N * (size_t)(K / 32 * 12);
     return 0;
@@ -179,7 +180,7 @@ logq_status logq_quantize(const float* W, int64_t N, int64_t K, int bits, double
 
     QuantParams p;
     memset(&p, 0, sizeof p);
-    for (int j = 0; j < 8; ++j) p.thresh[j] = cb.thresh[j];
+    for (int j = 0; j < 128; ++j) p.thresh[j] = cb.thresh[j];
     p.qmax = cb.qmax;
     p.bits = bits;
     p.check_nonfinite = auto_range ? 0 : 1;
@@ -240,7 +241,7 @@ logq_status logq_quantize_energy(const float* W, int64_t N, int64_t K, int bits,
     if (st_cb != LOGQ_OK) return st_cb;
     QuantParams p;
     memset(&p, 0, sizeof p);
-    for (int j = 0; j < 8; ++j) p.thresh[j] = cb.thresh[j];
+    for (int j = 0; j < 128; ++j) p.thresh[j] = cb.thresh[j];
     p.qmax = cb.qmax;
     p.bits = bits;
     p.check_nonfinite = 0;          // the range pass already looked at every weight

@@ -87,7 +87,7 @@ extern "C" logq_status logq_quantize_noalloc(const float* W, int64_t N, int64_t 
     if (st != LOGQ_OK) return st;
     QuantParams p;
     memset(&p, 0, sizeof p);
-    for (int j = 0; j < 8; ++j) p.thresh[j] = cb.thresh[j];
+    for (int j = 0; j < 128; ++j) p.thresh[j] = cb.thresh[j];
     p.qmax = cb.qmax;
     p.bits = bits;
     p.check_nonfinite = auto_range ? 0 : 1;

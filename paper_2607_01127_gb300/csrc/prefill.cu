@@ -702,6 +702,7 @@ constexpr uint32_t kSmemBytes = kTabRegion + kXStages * kXStageBytes + 256;
 
 cudaError_t launch_prefill(const LinearArgs& a, cudaStream_t s)
 {
+    if (a.bits != 3 && a.bits != 4) return cudaErrorNotSupported;   // 8-bit codes: decode path only
     auto encode = encode_fn();
     if (!encode) return cudaErrorNotSupported;
     CUtensorMap xmap;

@@ -183,6 +183,48 @@ __global__ void __launch_bounds__(256) quantize3_kernel(const float4* __restrict
     }
 }
 
+// 8-bit: each thread turns 16 consecutive weights into 16 code bytes.  The
+// 127 boundaries live in shared memory (as bit patterns, with +Inf appended)
+// and a seven-step binary search counts those not above |w|.
+__global__ void __launch_bounds__(256) quantize8_kernel(const float4* __restrict__ W, int64_t n16,
+                                                        QuantParams p, uint4* __restrict__ out,
+                                                        Workspace* ws)
+{
+    __shared__ uint32_t t[128];
+    if (threadIdx.x < 128) t[threadIdx.x] = threadIdx.x < 127 ? __float_as_uint(p.thresh[threadIdx.x]) : 0x7f800000u;
+    __syncthreads();
+    uint32_t umax = 0;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n16; i += stride) {
+        float4 v4[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) v4[j] = ld_stream(W + 4 * i + j);
+        uint32_t word[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const float v[4] = {v4[j].x, v4[j].y, v4[j].z, v4[j].w};
+            uint32_t wd = 0;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const uint32_t bits = __float_as_uint(v[e]);
+                const uint32_t u = bits & 0x7fffffffu;
+                umax = max(umax, u);
+                uint32_t m = 0;
+#pragma unroll
+                for (int step = 64; step >= 1; step >>= 1)
+                    if (u >= t[m + step - 1]) m += step;
+                wd |= code_of<8>(bits, m) << (8 * e);
+            }
+            word[j] = wd;
+        }
+        out[i] = make_uint4(word[0], word[1], word[2], word[3]);
+    }
+    if (p.check_nonfinite) {
+        const uint32_t bad = __reduce_or_sync(0xffffffffu, umax >= 0x7f800000u ? 1u : 0u);
+        if (bad && (threadIdx.x & 31) == 0) atomicOr(&ws->nonfinite, 1u);
+    }
+}
+
 int grid_for(int64_t items, int threads)
 {
     const int sms = sm_count() > 0 ? sm_count() : 148;
@@ -204,7 +246,11 @@ cudaError_t launch_quantize(const float* W, int64_t N, int64_t K, const QuantPar
                             uint8_t* codes, Workspace* ws, cudaStream_t s)
 {
     const int64_t total = N * K;
-    if (p.bits == 4) {
+    if (p.bits == 8) {
+        const int64_t n16 = total / 16;
+        quantize8_kernel<<<grid_for(n16, 256), 256, 0, s>>>(
+            reinterpret_cast<const float4*>(W), n16, p, reinterpret_cast<uint4*>(codes), ws);
+    } else if (p.bits == 4) {
         const int64_t nwords = total / 8;
         quantize4_kernel<<<grid_for(nwords, 256), 256, 0, s>>>(
             reinterpret_cast<const float4*>(W), nwords, p, reinterpret_cast<uint32_t*>(codes), ws);

@@ -38,12 +38,12 @@ def test_exports_every_declared_symbol(logq):
 
 
 def test_struct_layout_matches_header(logq):
-    # 4 int32 + 3 double + 16 float + 8 float + 2 x 16 uint16
-    assert ctypes.sizeof(logq.Codebook) == 16 + 24 + 64 + 32 + 64
+    # 4 int32 + 3 double + 256 float + 128 float + 2 x 256 uint16
+    assert ctypes.sizeof(logq.Codebook) == 16 + 24 + 1024 + 512 + 1024
 
 
-@pytest.mark.parametrize("bits", [3, 4])
-@pytest.mark.parametrize("base", [1.2, 1.25, 1.5, 1.7351, 2.0])
+@pytest.mark.parametrize("bits,base", [(b, x) for b in (3, 4) for x in (1.2, 1.25, 1.5, 1.7351, 2.0)]
+                         + [(8, x) for x in (1.02, 1.0473, 1.1)])
 @pytest.mark.parametrize("rng_", [0.0173, 0.31, 1.0, 2.75])
 @pytest.mark.parametrize("mode", [0, 1])
 def test_codebook_matches_oracle(logq, bits, base, rng_, mode):
@@ -81,7 +81,7 @@ def test_codebook_null_out(logq):
     assert logq.lib.logq_build_codebook(4, 1.5, 1.0, 0, None) == logq.LOGQ_ERR_INVALID_ARG
 
 
-@pytest.mark.parametrize("N,K,bits,want", [(512, 2048, 4, 512 * 1024), (3, 128, 3, 3 * 48),
+@pytest.mark.parametrize("N,K,bits,want", [(512, 2048, 4, 512 * 1024), (3, 128, 3, 3 * 48), (5, 256, 8, 5 * 256),
                                            (1, 128, 4, 64), (0, 128, 4, 0), (4, 100, 4, 0),
                                            (4, 0, 4, 0), (4, 128, 5, 0), (-1, 128, 4, 0),
                                            (14336, 4096, 3, 14336 * 1536)])
