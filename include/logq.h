@@ -155,8 +155,7 @@ logq_status logq_quantize(const float* W, int64_t N, int64_t K, int bits, double
  *   rounded to nearest-even.  All device pointers 16-byte aligned.
  *   B <= 16 (4-bit) or B <= 4 (3- and 8-bit) runs the decode GEMV /
  *   skinny-GEMM kernel on CUDA cores; larger B runs the prefill GEMM kernel
- *   on the tensor cores (tcgen05) for 3- and 4-bit codes and returns
- *   LOGQ_ERR_UNSUPPORTED for 8-bit codes.
+ *   on the tensor cores (tcgen05).
  * Asynchronous.  Errors: LOGQ_ERR_INVALID_ARG, LOGQ_ERR_UNSUPPORTED,
  * LOGQ_ERR_WORKSPACE, LOGQ_ERR_CUDA (launch).  A device-side wait that hit
  * its bound is reported later by logq_workspace_status. */

@@ -66,7 +66,6 @@ constexpr int kCodeStageBytes = kDecodeThreads * kCodeSlotBytes;
 constexpr uint32_t kTabOff = 1024;
 constexpr uint32_t kTabRow = 256;                // 32 lane copies in the first 128 bytes
 constexpr uint32_t kTabRegion = 256 * kTabRow;   // table rows (the 4-bit table uses all 256)
-static_assert(kCodeRing * kCodeStageBytes <= 256 * 128, "code ring must fit in the table rows' free halves");
 constexpr uint32_t kTmemCols = 512;              // accumulator (256) + weight stages (8 x 32)
 constexpr uint32_t kWCol0 = kBN;                 // first column of weight stage 0
 constexpr uint32_t kWStageCols = kBK / 2;        // 64 k of 16-bit values = 32 columns
@@ -89,7 +88,7 @@ struct PrefillParams {
     int32_t n_tiles_n, n_tiles_t;
     uint32_t idesc;
     uint32_t smem_bytes;    // dynamic shared memory of the launch (layout check)
-    uint32_t lvl16[16];
+    uint16_t lvl16[256];    // code-indexed 16-bit levels (2^bits used)
 };
 
 // ------------------------------------------------------------------ PTX ---
@@ -288,9 +287,17 @@ __device__ __forceinline__ void sts128(uint32_t addr, uint32_t a, uint32_t b, ui
 
 // ------------------------------------------------------------------ kernel ---
 
+// EIGHT: 8-bit codes, one per byte: a thread's 32 k of a stage are 32 bytes
+// (two ring slots), each byte resolves to one value (the table holds it in
+// both halves) and two values form a pair with one byte permute; the deeper
+// code footprint leaves room for RING = 3 stages in the table rows' halves.
+template <bool EIGHT>
 __global__ void __launch_bounds__(kThreads, 1)
 prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ CUtensorMap xmap)
 {
+    constexpr int SLOTS = EIGHT ? 2 : 1;                 // 16-byte ring slots per thread and stage
+    constexpr int RING = EIGHT ? 3 : kCodeRing;          // code stages in flight per decode thread
+    static_assert(RING * SLOTS * kCodeStageBytes <= 256 * 128, "code ring must fit in the table rows' free halves");
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     // Layout: pair table (code ring in its rows' free halves) | X stages | barriers
     const uint32_t sbase = smem_u32(smem_raw);
@@ -306,10 +313,11 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         }
         return;
     }
-    // code-ring slot of decode thread d in ring stage g: 16 bytes in the free
-    // half of table row g * 32 + d / 8
-    auto ring_slot = [&](int g, int d) -> uint32_t {
-        return sbase + (uint32_t)(g * (kDecodeThreads / 8) + (d >> 3)) * kTabRow + 128u + ((uint32_t)(d & 7) << 4);
+    // code-ring slot j of ring stage g: 16 bytes in the free half of table row
+    // g * 32 * SLOTS + j / 8 (decode thread d owns slots SLOTS * d .. +SLOTS-1)
+    auto ring_slot = [&](int g, int j) -> uint32_t {
+        return sbase + (uint32_t)(g * (SLOTS * kDecodeThreads / 8) + (j >> 3)) * kTabRow + 128u +
+               ((uint32_t)(j & 7) << 4);
     };
     uint8_t* gen = smem_raw - sbase;                  // generic pointer = gen + shared address
     // barriers: xfull[X], xempty[X], wfull[W], wempty[W], accfull, accempty, drain,
@@ -345,12 +353,17 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
     }
     // pair table: entry e (two codes) = bf16x2 / f16x2 of their levels, one copy per lane
     {
-        const int nent = (p.bits == 4) ? 256 : 64;
+        const int nent = (EIGHT || p.bits == 4) ? 256 : 64;
         for (int i = tid; i < nent * 8; i += kThreads) {
             const int e = i >> 3, part = i & 7;
-            const uint32_t lo = (p.bits == 4) ? (e & 15) : (e & 7);
-            const uint32_t hi = (p.bits == 4) ? (e >> 4) : (e >> 3);
-            const uint32_t v = (p.lvl16[lo] & 0xffffu) | (p.lvl16[hi] << 16);
+            uint32_t v;
+            if constexpr (EIGHT) {
+                v = (uint32_t)p.lvl16[e] * 0x10001u;
+            } else {
+                const uint32_t lo = (p.bits == 4) ? (e & 15) : (e & 7);
+                const uint32_t hi = (p.bits == 4) ? (e >> 4) : (e >> 3);
+                v = (uint32_t)p.lvl16[lo] | ((uint32_t)p.lvl16[hi] << 16);
+            }
             sts128(sbase + e * kTabRow + part * 16, v, v, v, v);
         }
     }
@@ -539,7 +552,7 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         const int h = dw >> 2;                          // half: k 32h .. 32h+31 of the stage
         const uint32_t tw = tmem_base + ((uint32_t)((warp & 3) * 32) << 16) + kWCol0 + (uint32_t)(16 * h);
         const uint32_t lane4 = 4u * (uint32_t)lane;
-        const int hbytes = (p.bits == 4) ? 16 : 12;     // codes of one half row per stage
+        const int hbytes = EIGHT ? 32 : (p.bits == 4) ? 16 : 12;   // codes of one half row per stage
         int stage = 0;
         uint32_t phase = 0;
         const int my_tiles = (ntiles > (int)blockIdx.x) ? (ntiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
@@ -567,8 +580,11 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         auto issue = [&](int g) {
             if (g < total && ahead.valid) {
                 const uint8_t* src = ahead.row + (int64_t)ahead.ks * (2 * hbytes);
-                const uint32_t dst = ring_slot(g % kCodeRing, d);
-                if (p.bits == 4) {
+                const uint32_t dst = ring_slot(g % RING, SLOTS * d);
+                if constexpr (EIGHT) {
+                    cp_async_16(dst, src);
+                    cp_async_16(dst + 16, src + 16);
+                } else if (p.bits == 4) {
                     cp_async_16(dst, src);
                 } else {
                     cp_async_4(dst, src);
@@ -581,6 +597,25 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         };
         // Resolve the codes of one stage (its slot in the ring) into 16 pair values.
         auto resolve = [&](int slot, bool valid, uint32_t (&pr)[16]) {
+            if constexpr (EIGHT) {
+                // word i holds the codes of k = 32h + 4i .. +3: pairs 2i and 2i + 1
+                uint4 c0 = make_uint4(0, 0, 0, 0), c1 = make_uint4(0, 0, 0, 0);
+                if (valid) {
+                    c0 = lds128(ring_slot(slot, SLOTS * d));
+                    c1 = lds128(ring_slot(slot, SLOTS * d) + 16);
+                }
+                const uint32_t cw8[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const uint32_t v0 = lds_tab(prmt(cw8[i], lane4, 0x7604u));
+                    const uint32_t v1 = lds_tab(prmt(cw8[i], lane4, 0x7614u));
+                    const uint32_t v2 = lds_tab(prmt(cw8[i], lane4, 0x7624u));
+                    const uint32_t v3 = lds_tab(prmt(cw8[i], lane4, 0x7634u));
+                    pr[2 * i] = prmt(v0, v1, 0x5410u);
+                    pr[2 * i + 1] = prmt(v2, v3, 0x5410u);
+                }
+                return;
+            }
             uint4 cv = make_uint4(0, 0, 0, 0);
             if (valid) cv = lds128(ring_slot(slot, d));
             const uint32_t cw[4] = {cv.x, cv.y, cv.z, cv.w};
@@ -609,12 +644,12 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         };
         // Software pipeline: the pairs of stage g+1 are looked up while stage g
         // waits for its weight slot and is stored.
-        for (int g = 0; g < kCodeRing - 1; ++g) issue(g);
+        for (int g = 0; g < RING - 1; ++g) issue(g);
         uint32_t pr_a[16], pr_b[16];
         int slot = 0;                                   // ring slot of stage g
         if (total > 0) {
-            issue(kCodeRing - 1);
-            cp_async_wait<kCodeRing - 1>();
+            issue(RING - 1);
+            cp_async_wait<RING - 1>();
             resolve(slot, cur.valid, pr_a);
             step(cur);
         }
@@ -623,10 +658,10 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         // buffers in alternating roles, so no pairs are copied.
         bool ok = true;
         auto stage_step = [&](int g, const uint32_t (&cur_pr)[16], uint32_t (&nxt_pr)[16]) {
-            if (++slot == kCodeRing) slot = 0;
+            if (++slot == RING) slot = 0;
             if (g + 1 < total) {
-                issue(g + kCodeRing);
-                cp_async_wait<kCodeRing - 1>();
+                issue(g + RING);
+                cp_async_wait<RING - 1>();
                 resolve(slot, cur.valid, nxt_pr);
                 step(cur);
             }
@@ -698,11 +733,33 @@ uint32_t make_idesc(bool f16_inputs)
 // Dynamic shared memory of the layout: table rows, X stages, barriers.
 constexpr uint32_t kSmemBytes = kTabRegion + kXStages * kXStageBytes + 256;
 
+template <bool EIGHT>
+cudaError_t launch(PrefillParams& p, const CUtensorMap& xmap, int grid, cudaStream_t s)
+{
+    static uint32_t configured[64] = {0};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    if (!configured[dev]) {
+        int reserved = 0, optin = 0;
+        if ((e = cudaDeviceGetAttribute(&reserved, cudaDevAttrReservedSharedMemoryPerBlock, dev)) != cudaSuccess) return e;
+        if ((e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev)) != cudaSuccess) return e;
+        const uint32_t bytes = kSmemBytes;
+        if (reserved != (int)kTabOff || bytes > (uint32_t)optin) return cudaErrorNotSupported;
+        e = cudaFuncSetAttribute(prefill_kernel<EIGHT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+        if (e != cudaSuccess) return e;
+        configured[dev] = bytes;
+    }
+    p.smem_bytes = configured[dev];
+    prefill_kernel<EIGHT><<<grid, kThreads, configured[dev], s>>>(p, xmap);
+    return cudaGetLastError();
+}
+
 }  // namespace
 
 cudaError_t launch_prefill(const LinearArgs& a, cudaStream_t s)
 {
-    if (a.bits != 3 && a.bits != 4) return cudaErrorNotSupported;   // 8-bit codes: decode path only
     auto encode = encode_fn();
     if (!encode) return cudaErrorNotSupported;
     CUtensorMap xmap;
@@ -726,34 +783,17 @@ cudaError_t launch_prefill(const LinearArgs& a, cudaStream_t s)
     p.K = (int32_t)a.K;
     p.B = (int32_t)a.B;
     p.bits = a.bits;
-    p.row_bytes = (a.bits == 4) ? a.K / 2 : a.K / 32 * 12;
+    p.row_bytes = (a.bits == 8) ? a.K : (a.bits == 4) ? a.K / 2 : a.K / 32 * 12;
     p.y_dtype = a.y_dtype;
     p.n_tiles_n = (int32_t)((a.N + kBM - 1) / kBM);
     p.n_tiles_t = (int32_t)((a.B + kBN - 1) / kBN);
     p.idesc = make_idesc(a.x_f16 != 0);
-    for (int c = 0; c < 16; ++c) p.lvl16[c] = a.lvl16[c];
+    for (int c = 0; c < (1 << a.bits); ++c) p.lvl16[c] = a.lvl16[c];
     const int64_t ntiles = (int64_t)p.n_tiles_n * p.n_tiles_t;
     const int sms = sm_count() > 0 ? sm_count() : 148;
     const int grid = (int)(ntiles < sms ? ntiles : sms);
 
-    static uint32_t configured[64] = {0};
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
-    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-    if (!configured[dev]) {
-        int reserved = 0, optin = 0;
-        if ((e = cudaDeviceGetAttribute(&reserved, cudaDevAttrReservedSharedMemoryPerBlock, dev)) != cudaSuccess) return e;
-        if ((e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev)) != cudaSuccess) return e;
-        const uint32_t bytes = kSmemBytes;
-        if (reserved != (int)kTabOff || bytes > (uint32_t)optin) return cudaErrorNotSupported;
-        e = cudaFuncSetAttribute(prefill_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
-        if (e != cudaSuccess) return e;
-        configured[dev] = bytes;
-    }
-    p.smem_bytes = configured[dev];
-    prefill_kernel<<<grid, kThreads, configured[dev], s>>>(p, xmap);
-    return cudaGetLastError();
+    return a.bits == 8 ? launch<true>(p, xmap, grid, s) : launch<false>(p, xmap, grid, s);
 }
 
 }  // namespace logq

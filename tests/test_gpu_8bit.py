@@ -1,8 +1,8 @@
 """8-bit Log_b codes (Sec. 3.1 with n = 8: q_max = 127, one code per byte)
 against the oracle: packed codes bit-exact (elements within one fp32 ulp of a
-boundary counted), decode GEMV outputs within 1e-3 * sum_k |x_k w_k| + 1e-6,
-self-calibrating range with the paper's 8-bit eps, and batches the 8-bit path
-does not cover rejected as unsupported."""
+boundary counted), decode GEMV and prefill GEMM outputs within
+1e-3 * sum_k |x_k w_k| + 1e-6, and the self-calibrating range with the
+paper's 8-bit eps."""
 import numpy as np
 import pytest
 import torch
@@ -126,10 +126,20 @@ def test_energy_range_8bit(logq):
     check_codes(codes.cpu().numpy(), w, ocb, 8)
 
 
-def test_batch_beyond_decode_path_unsupported(logq):
-    N, K = 64, 256
-    codes, cb = logq.logq_quantize(torch.from_numpy(workloads.weights_np(N, K, seed=5)).cuda(), 8, 1.05)
-    X = workloads.activations_torch(5, K, 6, torch.bfloat16, "cuda")
-    with pytest.raises(logq.LogqError) as ei:
-        logq.logq_linear(codes, cb, X, N, K)
-    assert ei.value.status == logq.LOGQ_ERR_UNSUPPORTED
+@pytest.mark.parametrize("N,K,B", [(64, 256, 5), (256, 512, 128), (300, 1152, 200), (1024, 2048, 256),
+                                   (512, 4096, 2048)])
+@pytest.mark.parametrize("ydt", [None, torch.bfloat16])
+def test_prefill8(logq, N, K, B, ydt):
+    """Batches above 4 run the tensor-core prefill with 8-bit codes (ragged
+    token tiles and weight-row tiles included)."""
+    w = workloads.weights_np(N, K, seed=N + K + B)
+    codes, cb = logq.logq_quantize(torch.from_numpy(w).cuda(), 8, 1.05)
+    ocb = oracle.build_codebook(8, 1.05, cb.range)
+    q = oracle.unpack(codes.cpu().numpy().reshape(N, -1), N, K, 8)
+    X = workloads.activations_torch(B, K, B, torch.bfloat16, "cuda")
+    ws = logq.new_workspace()
+    Y = logq.logq_linear(codes, cb, X, N, K, y_dtype=ydt, workspace=ws)
+    Yr, A = reference(X, q, ocb)
+    check_linear(Y.double().cpu().numpy(), Yr, A, "f32" if ydt is None else "bf16")
+    st, _ = logq.logq_workspace_status(ws)
+    assert st == logq.LOGQ_OK
