@@ -61,8 +61,9 @@ def model_layers():
     return out
 
 
-def linear_bytes(N, K, B=1, bits=4):
-    return N * K * bits // 8 + B * K * 2 + B * N * 4
+def linear_bytes(N, K, B=1, bits=4, y_bytes=4):
+    """Algorithmic bytes of one linear: packed codes, bf16 activations, outputs."""
+    return N * K * bits // 8 + B * K * 2 + B * N * y_bytes
 
 
 class ClockSampler:
@@ -156,7 +157,7 @@ def oracle_gemv_run(items, threads: int):
         bs = np.zeros(R, np.int64)
         ns = np.arange(R, dtype=np.int64)
         oracle.linear_sampled(x, packed, 4, cb, oracle.TABLE_BF16, bs, ns, nthreads=threads)
-        nbytes += linear_bytes(R, K)
+        nbytes += linear_bytes(R, K, y_bytes=2)      # same per-output bytes as the device step
     return nbytes
 
 
@@ -249,7 +250,8 @@ def build_decode_model(logq, torch, dev):
 
 
 def linear_bytes_of(launch):
-    return sum(linear_bytes(m["N"], m["K"]) for m in launch["members"])
+    # the chained step writes bf16 outputs (2 bytes each)
+    return sum(linear_bytes(m["N"], m["K"], y_bytes=2) for m in launch["members"])
 
 
 def time_quantize(logq, torch, dev, reps: int = 2):
@@ -288,6 +290,56 @@ def time_energy(logq, torch, dev, reps: int = 5):
         logq.logq_quantize_energy(W, 4, 4e-3, codes=codes, workspace=ws, scratch=scratch)
     dt = (time.perf_counter() - t0) / reps          # the call synchronises twice
     return {"us": dt * 1e6, "weights": N * K, "wmin": wmin, "base": cb.base, "range": cb.range}
+
+
+def time_8bit(logq, torch, dev, reps: int = 10):
+    """8-bit codes (q_max = 127) on the Llama-3.1-8B gate shape: the batch-1 decode GEMV over
+    rotating copies of the codes (more than L2 holds), and the 2048-token prefill GEMM."""
+    N, K = workloads.LLAMA_8B_SHAPES["gate"]
+    ws = logq.new_workspace(dev)
+    W = workloads.weights_torch(N, K, workloads.layer_seed(4, 0, 4), outliers=True, device=dev)
+    codes, cb = logq.logq_quantize(W, 8, 1.04, workspace=ws)
+    del W
+    copies = [codes] + [codes.clone() for _ in range(11)]          # 12 x 58.7 MB
+    X = workloads.activations_torch(1, K, 3, torch.bfloat16, dev)
+    Y = torch.empty(1, N, dtype=torch.bfloat16, device=dev)
+    s = torch.cuda.Stream(dev)
+    def launches():
+        for c in copies:
+            logq.logq_linear(c, cb, X, N, K, y_dtype=torch.bfloat16, Y=Y, workspace=ws)
+    with torch.cuda.stream(s):
+        launches()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(s):
+        with torch.cuda.graph(g, stream=s):
+            launches()
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()                                     # replays run on the current stream
+    for _ in range(reps):
+        g.replay()
+    e1.record()
+    torch.cuda.synchronize()
+    t = e0.elapsed_time(e1) * 1e-3 / (reps * len(copies))
+    nbytes = linear_bytes(N, K, bits=8, y_bytes=2)
+    del copies
+    Xp = workloads.activations_torch(PREFILL_TOKENS, K, 4, torch.bfloat16, dev)
+    Yp = torch.empty(PREFILL_TOKENS, N, dtype=torch.bfloat16, device=dev)
+    logq.logq_linear(codes, cb, Xp, N, K, y_dtype=torch.bfloat16, Y=Yp, workspace=ws)
+    torch.cuda.synchronize()
+    e0.record()
+    for _ in range(3):
+        logq.logq_linear(codes, cb, Xp, N, K, y_dtype=torch.bfloat16, Y=Yp, workspace=ws)
+    e1.record()
+    torch.cuda.synchronize()
+    tp = e0.elapsed_time(e1) * 1e-3 / 3
+    st, _ = logq.logq_workspace_status(ws)
+    assert st == logq.LOGQ_OK
+    return {"gemv_us": t * 1e6, "gemv_gbs": nbytes / t / 1e9, "gemv_bytes": nbytes,
+            "prefill_us": tp * 1e6, "prefill_tflops": 2.0 * PREFILL_TOKENS * N * K / tp / 1e12}
 
 
 def time_prefill(logq, torch, dev, reps: int = 3):
@@ -495,6 +547,17 @@ def run_ours(args):
         except Exception as e:
             line["energy_quantize"] = {"error": str(e)[:200]}
         try:
+            e8 = time_8bit(logq, torch, dev)
+            line["bits8"] = {
+                "gemv_us": round(e8["gemv_us"], 2), "gemv_gbs": round(e8["gemv_gbs"], 1),
+                "gemv_frac": round(e8["gemv_gbs"] / pk["hbm_gbs"], 4),
+                "prefill_tflops": round(e8["prefill_tflops"], 1),
+                "prefill_frac": round(e8["prefill_tflops"] / pk["bf16_tflops"], 4),
+                "note": "8-bit codes, Llama-3.1-8B gate 14336x4096: batch-1 decode GEMV over 12 rotating "
+                        "copies of the codes (0.70 GB, beyond L2), bf16 output; prefill with 2048 tokens"}
+        except Exception as e:
+            line["bits8"] = {"error": str(e)[:200]}
+        try:
             pf = time_prefill(logq, torch, dev)
             if pf is not None:
                 line["prefill"] = {"tflops": round(pf["tflops"], 1), "unit": "TFLOP/s",
@@ -513,7 +576,8 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
-CASES = ("gemv_gateup_1b", "gemv_gate_8b", "prefill_q_8b", "quantize_gate_8b", "energy_gate_8b")
+CASES = ("gemv_gateup_1b", "gemv_gate_8b", "prefill_q_8b", "quantize_gate_8b", "energy_gate_8b",
+         "gemv8_gate_8b")
 
 
 def run_case(name: str):
@@ -549,6 +613,12 @@ def run_case(name: str):
         W = workloads.weights_torch(N, K, 15, True, dev)
         for _ in range(2):
             logq.logq_quantize(W, 4, 1.5, workspace=ws)
+    elif name == "gemv8_gate_8b":
+        N, K = workloads.LLAMA_8B_SHAPES["gate"]
+        c = logq.logq_quantize(workloads.weights_torch(N, K, 13, True, dev), 8, 1.04, workspace=ws)
+        X = workloads.activations_torch(1, K, 1, torch.bfloat16, dev)
+        for _ in range(2):
+            logq.logq_linear(c[0], c[1], X, N, K, workspace=ws)
     elif name == "energy_gate_8b":
         N, K = workloads.LLAMA_8B_SHAPES["gate"]
         W = workloads.weights_torch(N, K, 15, True, dev)
