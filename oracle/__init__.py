@@ -20,6 +20,9 @@ Parity status of each function (what pins it is in ``tests/test_oracle.py``):
   linear               pinned (float64 matmul of the dequantised weights,
                         one-hot and zero inputs)
   energy_wmin          pinned (brute force over all candidate thresholds)
+  gptq                 pinned (diagonal Hessian = plain rounding; every compensated
+                        value equals the least-squares minimiser given the columns
+                        already quantised, solved directly)
   base_from_range      pinned (closed form: q_max log steps span the range)
 """
 from __future__ import annotations
@@ -141,6 +144,8 @@ def _load():
     lib.oracle_energy_wmin.restype = c_dbl
     lib.oracle_base_from_range.argtypes = [c_dbl, c_dbl, c_int]
     lib.oracle_base_from_range.restype = c_dbl
+    lib.oracle_gptq.argtypes = [P, c_i64, c_i64, P, c_dbl, ctypes.POINTER(Codebook), P, P]
+    lib.oracle_gptq.restype = c_int
     _lib = lib
     return lib
 
@@ -247,6 +252,20 @@ def linear_sampled(X: np.ndarray, packed: np.ndarray, bits: int, cb: Codebook, t
                                   int(table), _ptr(bs), _ptr(ns), bs.size, _ptr(Y), _ptr(A),
                                   int(nthreads))
     return Y, A
+
+
+def gptq(w, H, cb: Codebook, damp: float = 0.01):
+    """GPTQ with the Log_b quantiser (fp64, column by column).  Returns the signed
+    codes and the value each weight had when its column was quantised."""
+    w = _f32(w)
+    N, K = w.shape
+    H = np.ascontiguousarray(H, dtype=np.float64)
+    q = np.empty((N, K), dtype=np.int8)
+    w_at = np.empty((N, K), dtype=np.float64)
+    rc = _load().oracle_gptq(_ptr(w), N, K, _ptr(H), float(damp), ctypes.byref(cb), _ptr(q), _ptr(w_at))
+    if rc != 0:
+        raise ValueError("gptq: damped Hessian is not positive definite")
+    return q, w_at
 
 
 def round_f32(v: float) -> float:

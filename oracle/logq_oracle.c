@@ -477,3 +477,95 @@ double oracle_base_from_range(double wmax, double wmin, int bits)
     if (!(wmax > 0.0) || !(wmin > 0.0) || qmax < 1) return -1.0;
     return pow(wmax / wmin, 1.0 / (double)qmax);
 }
+
+/* ---- GPTQ with the Log_b quantiser (Sec. 3.3 uses GPTQ for calibration) --- */
+/*
+ * The published GPTQ procedure, column by column in fp64:
+ *   Hd = H + damp * mean(diag H) * I   (a zero diagonal entry becomes 1 and its
+ *        weight column 0: the column never sees input),
+ *   Hd^-1 = U^T U with U upper triangular (Cholesky of the inverse),
+ *   for j = 0 .. K-1:  q_j = Quant(w_j) (decision boundaries, R3),
+ *                      e_j = (w_j - level32(q_j)) / U_jj,
+ *                      w_c -= e_j * U_jc  for every later column c.
+ * w_at[r][j] receives the value of w_j when column j was quantised.  The
+ * quantiser's value for the error is the fp32 level (R5).  Returns 0 on
+ * success, 1 when Hd is not positive definite.
+ */
+static int chol_lower(double* A, int64_t n)          /* A = L L^T in place (lower) */
+{
+    for (int64_t j = 0; j < n; ++j) {
+        double d = A[j * n + j];
+        for (int64_t k = 0; k < j; ++k) d -= A[j * n + k] * A[j * n + k];
+        if (!(d > 0.0)) return 1;
+        d = sqrt(d);
+        A[j * n + j] = d;
+        for (int64_t i = j + 1; i < n; ++i) {
+            double s = A[i * n + j];
+            for (int64_t k = 0; k < j; ++k) s -= A[i * n + k] * A[j * n + k];
+            A[i * n + j] = s / d;
+        }
+        for (int64_t i = 0; i < j; ++i) A[i * n + j] = 0.0;
+    }
+    return 0;
+}
+
+int oracle_gptq(const float* W, int64_t N, int64_t K, const double* H, double damp,
+                const oracle_codebook* cb, int8_t* q, double* w_at)
+{
+    double* A = (double*)malloc(sizeof(double) * (size_t)(K * K));
+    double* Hinv = (double*)malloc(sizeof(double) * (size_t)(K * K));
+    double* w = (double*)malloc(sizeof(double) * (size_t)(N * K));
+    int rc = 1;
+    double mean = 0.0;
+    for (int64_t j = 0; j < K; ++j) mean += H[j * K + j];
+    mean /= (double)K;
+    memcpy(A, H, sizeof(double) * (size_t)(K * K));
+    for (int64_t i = 0; i < N * K; ++i) w[i] = (double)W[i];
+    for (int64_t j = 0; j < K; ++j) {
+        if (H[j * K + j] == 0.0) {
+            A[j * K + j] = 1.0;
+            for (int64_t r = 0; r < N; ++r) w[r * K + j] = 0.0;
+        }
+        A[j * K + j] += damp * mean;
+    }
+    /* Hd = L L^T; Hd^-1 column by column from L y = e_c, L^T x = y */
+    if (chol_lower(A, K)) goto out;
+    for (int64_t c = 0; c < K; ++c) {
+        for (int64_t i = 0; i < K; ++i) {                 /* forward */
+            double s = (i == c) ? 1.0 : 0.0;
+            for (int64_t k = 0; k < i; ++k) s -= A[i * K + k] * Hinv[k * K + c];
+            Hinv[i * K + c] = s / A[i * K + i];
+        }
+        for (int64_t i = K - 1; i >= 0; --i) {            /* backward */
+            double s = Hinv[i * K + c];
+            for (int64_t k = i + 1; k < K; ++k) s -= A[k * K + i] * Hinv[k * K + c];
+            Hinv[i * K + c] = s / A[i * K + i];
+        }
+    }
+    /* Hd^-1 = U^T U: U = (lower Cholesky factor of Hd^-1)^T */
+    if (chol_lower(Hinv, K)) goto out;
+    for (int64_t r = 0; r < N; ++r) {
+        double* wr = w + r * K;
+        for (int64_t j = 0; j < K; ++j) {
+            double x = wr[j];
+            if (w_at) w_at[r * K + j] = x;
+            double a = fabs(x);
+            int m = 0;
+            for (int t = 0; t < cb->qmax; ++t)
+                if (a >= cb->tau[t]) m++;
+            int8_t qv = (int8_t)(x < 0 ? -m : m);
+            q[r * K + j] = qv;
+            double deq = (qv < 0 ? -1.0 : 1.0) * (double)cb->level32[m];
+            if (m == 0) deq = 0.0;
+            double ujj = Hinv[j * K + j];                  /* U_jj = L^T_jj */
+            double e = (x - deq) / ujj;
+            for (int64_t c = j + 1; c < K; ++c) wr[c] -= e * Hinv[c * K + j];   /* U_jc = L_cj */
+        }
+    }
+    rc = 0;
+out:
+    free(A);
+    free(Hinv);
+    free(w);
+    return rc;
+}

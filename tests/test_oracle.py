@@ -322,3 +322,55 @@ def test_base_from_range_spans_qmax_steps(bits):
     # b^(0 - s), which Eq. (2) maps to zero) up to w_max = L_qmax
     assert math.isclose(b ** (0 - cb.shift), wmin, rel_tol=1e-12)
     assert math.isclose(cb.levels[1], wmin * b, rel_tol=1e-12)
+
+
+# ------------------------------------------------------------ GPTQ ---
+
+def _hessian(K, seed, T=None):
+    rng = np.random.Generator(np.random.PCG64(seed))
+    X = rng.standard_normal((T or 4 * K, K)) * (1.0 + rng.random(K))   # correlated-free, varied scales
+    X[:, 1:] += 0.5 * X[:, :-1]                                        # neighbouring inputs correlate
+    return X.T @ X
+
+
+@pytest.mark.parametrize("bits", [4, 8])
+def test_gptq_diagonal_hessian_is_plain_rounding(bits):
+    """With a diagonal Hessian no column informs another: GPTQ = rounding to nearest."""
+    w = workloads.weights_np(16, 64, 8)
+    cb = oracle.build_codebook(bits, 1.5 if bits == 4 else 1.05, float(np.abs(w).max()))
+    H = np.diag(np.random.Generator(np.random.PCG64(1)).random(64) + 0.5)
+    q, w_at = oracle.gptq(w, H, cb)
+    np.testing.assert_array_equal(q, oracle.quantize_thresh(w, cb))
+    np.testing.assert_array_equal(w_at, w.astype(np.float64))
+
+
+@pytest.mark.parametrize("bits", [4, 8])
+@pytest.mark.parametrize("K", [2, 7, 24])
+def test_gptq_compensation_is_least_squares(bits, K):
+    """The value column j is quantised at is the j-th entry of the minimiser of
+    (x - w) Hd (x - w)^T with the earlier columns fixed at their levels --
+    solved here directly, without the Cholesky route the oracle takes."""
+    N, damp = 5, 0.01
+    w = workloads.weights_np(N, K, 9 + K)
+    cb = oracle.build_codebook(bits, 1.4 if bits == 4 else 1.05, float(np.abs(w).max()))
+    H = _hessian(K, K)
+    q, w_at = oracle.gptq(w, H, cb, damp)
+    Hd = H + damp * np.mean(np.diag(H)) * np.eye(K)
+    deq = oracle.dequant(q, cb, oracle.TABLE_F32)
+    wd = w.astype(np.float64)
+    for j in range(1, K):
+        d, r = slice(0, j), slice(j, K)
+        delta = deq[:, d] - wd[:, d]                                  # fixed changes of done columns
+        x_r = wd[:, r] - np.linalg.solve(Hd[r, r], Hd[r, d] @ delta.T).T
+        np.testing.assert_allclose(w_at[:, j], x_r[:, 0], rtol=1e-9, atol=1e-12)
+
+
+def test_gptq_lowers_the_layer_loss():
+    """tr((W - What) Hd (W - What)^T) below that of plain rounding on correlated inputs."""
+    w = workloads.weights_np(32, 96, 12)
+    cb = oracle.build_codebook(4, 1.5, float(np.abs(w).max()))
+    H = _hessian(96, 3)
+    q, _ = oracle.gptq(w, H, cb)
+    loss = lambda qq: float(np.trace((w - oracle.dequant(qq, cb, oracle.TABLE_F32)) @ H @
+                                     (w - oracle.dequant(qq, cb, oracle.TABLE_F32)).T))
+    assert loss(q) < 0.9 * loss(oracle.quantize_thresh(w, cb))
