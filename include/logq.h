@@ -221,6 +221,36 @@ logq_status logq_quantize_energy(const float* W, int64_t N, int64_t K, int bits,
                                  void* workspace, size_t workspace_bytes, void* scratch,
                                  size_t scratch_bytes, void* stream);
 
+/* Bytes of device scratch logq_gptq needs for an N x K matrix (the working copy
+ * of W plus the errors of one 128-column block); 0 for invalid sizes. */
+size_t logq_gptq_scratch_bytes(int64_t N, int64_t K);
+
+/*
+ * GPTQ with the Log_b quantiser: the post-training calibration the paper
+ * quantises its models with (Sec. 3.3 / Sec. 4, GPTQ's published procedure).
+ * The columns of W are quantised in order with the codebook cb (Eq. (1) as
+ * m = #{ j : |w| >= thresh[j] }); after column j the error
+ * e = (w_j - level(q_j)) / U[j][j] (level = the fp32 level of the code) is
+ * compensated on every later column c: w_c -= e * U[j][c].  Processed in
+ * blocks of 128 columns; the columns after a block receive the block's
+ * compensation as one product.
+ *   W (device, fp32, [N][K], 16-byte aligned): not modified.
+ *   U (device, fp32, [K][K] row-major): the upper Cholesky factor of the damped
+ *     inverse Hessian, Hd^-1 = U^T U (Hd = H + damping, H = 2 X^T X of the
+ *     layer's inputs); only the upper triangle is read.  Columns whose Hessian
+ *     diagonal is zero should be zeroed in W by the caller (they never see input).
+ *   cb (host): the codebook (bits 4 or 8), e.g. from logq_build_codebook with
+ *     the range and base of the original W.
+ *   codes (device): logq_packed_bytes(N, K, bits) bytes, the packed result.
+ *   scratch: logq_gptq_scratch_bytes(N, K) bytes of device memory.
+ * Asynchronous (a device copy and 2 K / 128 - 1 launches on `stream`).
+ * Errors: LOGQ_ERR_INVALID_ARG (sizes, pointers, alignment, codebook),
+ * LOGQ_ERR_UNSUPPORTED (3-bit codebooks), LOGQ_ERR_WORKSPACE (scratch),
+ * LOGQ_ERR_CUDA.
+ */
+logq_status logq_gptq(const float* W, int64_t N, int64_t K, const float* U, const logq_codebook* cb,
+                      uint8_t* codes, void* scratch, size_t scratch_bytes, void* stream);
+
 /* One matrix of logq_linear_grouped. */
 typedef struct logq_linear_item {
     const uint8_t* codes;       /* device: packed codes of this matrix, N rows */

@@ -16,7 +16,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "liblogq.so")
-SOURCES = ["logq_host.cu", "quantize.cu", "energy.cu", "gemv.cu", "prefill.cu", "noalloc.cu"]
+SOURCES = ["logq_host.cu", "quantize.cu", "energy.cu", "gptq.cu", "gemv.cu", "prefill.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

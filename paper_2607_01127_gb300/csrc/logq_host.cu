@@ -252,6 +252,27 @@ logq_status logq_quantize_energy(const float* W, int64_t N, int64_t K, int bits,
     return LOGQ_OK;
 }
 
+size_t logq_gptq_scratch_bytes(int64_t N, int64_t K)
+{
+    if (N <= 0 || K <= 0 || (K % 128) != 0) return 0;
+    return gptq_scratch_bytes(N, K);
+}
+
+logq_status logq_gptq(const float* W, int64_t N, int64_t K, const float* U, const logq_codebook* cb,
+                      uint8_t* codes, void* scratch, size_t scratch_bytes, void* stream)
+{
+    if (!W || !U || !cb || !codes) return LOGQ_ERR_INVALID_ARG;
+    if (!aligned16(W) || !aligned16(U) || !aligned16(codes)) return LOGQ_ERR_INVALID_ARG;
+    if (logq_packed_bytes(N, K, cb->bits) == 0) return LOGQ_ERR_INVALID_ARG;
+    if (cb->qmax != (1 << (cb->bits - 1)) - 1) return LOGQ_ERR_INVALID_ARG;
+    if (N > (int64_t(1) << 40) / K) return LOGQ_ERR_INVALID_ARG;
+    if (cb->bits != 4 && cb->bits != 8) return LOGQ_ERR_UNSUPPORTED;
+    if (!scratch || !aligned16(scratch) || scratch_bytes < gptq_scratch_bytes(N, K)) return LOGQ_ERR_WORKSPACE;
+    const cudaError_t e = launch_gptq(W, N, K, U, cb->bits, cb->thresh, cb->level, cb->qmax, codes, scratch,
+                                      static_cast<cudaStream_t>(stream));
+    return cuda_status(e);
+}
+
 logq_status logq_linear(const uint8_t* codes, const logq_codebook* cb, const void* X,
                         logq_dtype x_dtype, int64_t B, int64_t N, int64_t K, void* Y,
                         logq_dtype y_dtype, void* workspace, size_t workspace_bytes, void* stream)

@@ -160,6 +160,27 @@ def test_energy_quantize_rejects_before_launch(logq):
     assert call(sc=_fake(0x40004)) == logq.LOGQ_ERR_WORKSPACE
 
 
+def test_gptq_rejects_before_launch(logq):
+    """logq_gptq validates sizes, codebook and scratch before anything is enqueued."""
+    L = logq.lib
+    W, U, C, sc = _fake(0x10000), _fake(0x20000), _fake(0x30000), _fake(0x40000)
+    cb4 = logq.logq_build_codebook(4, 1.5, 1.0)
+    cb3 = logq.logq_build_codebook(3, 1.5, 1.0)
+    scb = L.logq_gptq_scratch_bytes(64, 256)
+    assert scb == (64 * 256 + 64 * 128) * 4
+    assert L.logq_gptq_scratch_bytes(64, 100) == 0
+
+    def call(W=W, U=U, cb=cb4, C=C, sc=sc, scb=scb, N=64, K=256):
+        return L.logq_gptq(W, N, K, U, ctypes.byref(cb), C, sc, scb, None)
+
+    assert call(W=None) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(U=_fake(0x20004)) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(K=100) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(cb=cb3) == logq.LOGQ_ERR_UNSUPPORTED
+    assert call(sc=None) == logq.LOGQ_ERR_WORKSPACE
+    assert call(scb=scb - 16) == logq.LOGQ_ERR_WORKSPACE
+
+
 def test_linear_rejects_before_launch(logq):
     L = logq.lib
     cb = logq.logq_build_codebook(4, 1.5, 1.0)
