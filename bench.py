@@ -342,6 +342,57 @@ def time_8bit(logq, torch, dev, reps: int = 10):
             "prefill_us": tp * 1e6, "prefill_tflops": 2.0 * PREFILL_TOKENS * N * K / tp / 1e12}
 
 
+def time_gptq(logq, torch, dev):
+    """GPTQ with the Log_b quantiser on the Llama-3.1-8B q shape (4096 x 4096): Hessian of
+    3 K synthetic tokens (neighbouring inputs correlated), the self-calibrated 4-bit codebook;
+    the device time of the factor (logq_gptq_factor) and of the quantisation (logq_gptq),
+    and the layer loss tr((W - What) H (W - What)^T) against plain rounding with the same
+    codebook."""
+    import ctypes
+    N, K = workloads.LLAMA_8B_SHAPES["q"]
+    W = workloads.weights_torch(N, K, workloads.layer_seed(4, 0, 0), outliers=True, device=dev)
+    g = torch.Generator(device=dev).manual_seed(CFG_SEED)
+    X = torch.randn(3 * K, K, device=dev, generator=g, dtype=torch.float64)
+    X[:, 1:] += 0.5 * X[:, :-1].clone()
+    H64 = X.T @ X
+    del X
+    H = H64.float()
+    rtn, cb, _ = logq.logq_quantize_energy(W, 4, 4e-3)
+    U = torch.empty(K, K, device=dev)
+    dead = torch.empty(K, dtype=torch.uint8, device=dev)
+    fscratch = torch.empty(int(logq._lib().logq_gptq_factor_scratch_bytes(K)), dtype=torch.uint8, device=dev)
+    codes = torch.empty(N * K // 2, dtype=torch.uint8, device=dev)
+    scratch = torch.empty(int(logq._lib().logq_gptq_scratch_bytes(N, K)), dtype=torch.uint8, device=dev)
+    def factor():
+        logq.gptq_factor(H, 0.01, U=U, dead=dead, scratch=fscratch)
+    def run():
+        st = logq._lib().logq_gptq(ctypes.c_void_p(W.data_ptr()), N, K, ctypes.c_void_p(U.data_ptr()),
+                                   ctypes.c_void_p(dead.data_ptr()), ctypes.byref(cb),
+                                   ctypes.c_void_p(codes.data_ptr()), ctypes.c_void_p(scratch.data_ptr()),
+                                   scratch.numel(), None)
+        assert st == logq.LOGQ_OK
+    def timed(fn):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        fn()
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1)
+    factor()
+    run()
+    torch.cuda.synchronize()
+    factor_ms = timed(factor)
+    ms = timed(run)
+    lv = torch.tensor(list(cb.level[:16]), dtype=torch.float64, device=dev)
+    def loss(c):
+        b = c.view(N, K // 2)
+        d = W.double() - lv[torch.stack([b & 15, b >> 4], dim=-1).view(N, K).long()]
+        return float(((d @ H64) * d).sum())
+    upd = sum(2 * N * 128 * (K - j0 - 128) for j0 in range(0, K, 128))
+    return {"ms": ms, "factor_ms": factor_ms, "update_tflops": upd / (ms * 1e-3) / 1e12,
+            "loss_ratio": loss(codes) / loss(rtn)}
+
+
 def time_prefill(logq, torch, dev, reps: int = 3):
     """Prefill GEMM: 2048 tokens x each Llama-3.1-8B linear shape."""
     res = {}
@@ -558,6 +609,17 @@ def run_ours(args):
         except Exception as e:
             line["bits8"] = {"error": str(e)[:200]}
         try:
+            gq = time_gptq(logq, torch, dev)
+            line["gptq"] = {"ms": round(gq["ms"], 2), "factor_ms": round(gq["factor_ms"], 1),
+                            "update_tflops": round(gq["update_tflops"], 2),
+                            "loss_vs_rounding": round(gq["loss_ratio"], 4),
+                            "note": "4-bit GPTQ of a Llama-3.1-8B q matrix (4096x4096), Hessian of 12288 synthetic "
+                                    "tokens, self-calibrated codebook; ms = logq_gptq (column blocks + fp32 "
+                                    "updates), factor_ms = logq_gptq_factor (fp32 Cholesky + triangular inverse, "
+                                    "one host sync)"}
+        except Exception as e:
+            line["gptq"] = {"error": str(e)[:200]}
+        try:
             pf = time_prefill(logq, torch, dev)
             if pf is not None:
                 line["prefill"] = {"tflops": round(pf["tflops"], 1), "unit": "TFLOP/s",
@@ -577,14 +639,15 @@ def run_ours(args):
 
 
 CASES = ("gemv_gateup_1b", "gemv_gate_8b", "prefill_q_8b", "quantize_gate_8b", "energy_gate_8b",
-         "gemv8_gate_8b")
+         "gemv8_gate_8b", "gptq_q_8b")
 
 
 def run_case(name: str):
     """One small workload run twice (for a profiler capture of the second run):
     the gate+up launch of the 1B decode step, the 8B gate GEMV, the 8B q-shaped
-    prefill GEMM (2048 tokens), the quantisation of an 8B gate matrix and its
-    self-calibrating (energy-range) quantisation."""
+    prefill GEMM (2048 tokens), the quantisation of an 8B gate matrix, its
+    self-calibrating (energy-range) quantisation, the 8-bit gate GEMV and 4-bit
+    GPTQ of an 8B q matrix (factor and quantisation)."""
     import torch
     import paper_2607_01127_gb300 as logq
     dev = torch.device("cuda", 0)
@@ -624,6 +687,16 @@ def run_case(name: str):
         W = workloads.weights_torch(N, K, 15, True, dev)
         for _ in range(2):
             logq.logq_quantize_energy(W, 4, 4e-3, workspace=ws)
+    elif name == "gptq_q_8b":
+        N, K = workloads.LLAMA_8B_SHAPES["q"]
+        W = workloads.weights_torch(N, K, 16, True, dev)
+        g = torch.Generator(device=dev).manual_seed(17)
+        X = torch.randn(2 * K, K, device=dev, generator=g)
+        H = X.T @ X
+        del X
+        cb = logq.logq_build_codebook(4, 1.5, float(W.abs().max()))
+        for _ in range(2):
+            logq.logq_gptq(W, H, cb)
     torch.cuda.synchronize()
     st, _ = logq.logq_workspace_status(ws)
     assert st == logq.LOGQ_OK

@@ -57,7 +57,8 @@ typedef enum {
     LOGQ_ERR_UNSUPPORTED = 3,   /* valid request the library does not implement */
     LOGQ_ERR_CUDA = 4,          /* a CUDA runtime call or launch failed */
     LOGQ_ERR_WORKSPACE = 5,     /* workspace missing, too small or misaligned */
-    LOGQ_ERR_TIMEOUT = 6        /* a device-side pipeline wait hit its bound */
+    LOGQ_ERR_TIMEOUT = 6,       /* a device-side pipeline wait hit its bound */
+    LOGQ_ERR_NOT_PD = 7         /* logq_gptq_factor: the damped Hessian is not positive definite */
 } logq_status;
 
 typedef enum {
@@ -221,6 +222,34 @@ logq_status logq_quantize_energy(const float* W, int64_t N, int64_t K, int bits,
                                  void* workspace, size_t workspace_bytes, void* scratch,
                                  size_t scratch_bytes, void* stream);
 
+/* Bytes of device scratch logq_gptq_factor needs for a K x K Hessian (1.25 K^2
+ * floats and 256 bytes); 0 for invalid K. */
+size_t logq_gptq_factor_scratch_bytes(int64_t K);
+
+/*
+ * The factor GPTQ compensates with (GPTQ's published procedure, the
+ * calibration the paper quantises its models with, Sec. 3.3 / Sec. 4):
+ * Hd = H + damp * mean(diag H) * I, a zero diagonal entry of H (an input that
+ * never fires) set to 1 first; U = the upper Cholesky factor of Hd^-1
+ * (Hd^-1 = U^T U), computed in fp32 on the device as the inverse of the
+ * index-reversed Cholesky factor of Hd.
+ *   H (device, fp32, [K][K] row-major, symmetric, 16-byte aligned): e.g.
+ *     2 X^T X of the layer's calibration inputs; K a multiple of 128, at most
+ *     65536.  Not modified.
+ *   damp: finite, >= 0 (GPTQ's usual value is 0.01).
+ *   U (device, fp32, [K][K], 16-byte aligned): receives the factor, zeros
+ *     below the diagonal.
+ *   dead (device, K bytes, may be NULL): receives 1 for every input whose
+ *     Hessian diagonal is zero, else 0 -- hand it to logq_gptq.
+ *   scratch: logq_gptq_factor_scratch_bytes(K) bytes of device memory.
+ * Synchronises `stream` once (to read the positive-definiteness flag).
+ * Errors: LOGQ_ERR_INVALID_ARG (sizes, pointers, alignment, damp),
+ * LOGQ_ERR_WORKSPACE (scratch), LOGQ_ERR_NOT_PD (a Cholesky pivot was not
+ * positive or not finite: U is then unspecified), LOGQ_ERR_CUDA.
+ */
+logq_status logq_gptq_factor(const float* H, int64_t K, double damp, float* U, uint8_t* dead, void* scratch,
+                             size_t scratch_bytes, void* stream);
+
 /* Bytes of device scratch logq_gptq needs for an N x K matrix (the working copy
  * of W plus the errors of one 128-column block); 0 for invalid sizes. */
 size_t logq_gptq_scratch_bytes(int64_t N, int64_t K);
@@ -234,11 +263,14 @@ size_t logq_gptq_scratch_bytes(int64_t N, int64_t K);
  * compensated on every later column c: w_c -= e * U[j][c].  Processed in
  * blocks of 128 columns; the columns after a block receive the block's
  * compensation as one product.
- *   W (device, fp32, [N][K], 16-byte aligned): not modified.
- *   U (device, fp32, [K][K] row-major): the upper Cholesky factor of the damped
- *     inverse Hessian, Hd^-1 = U^T U (Hd = H + damping, H = 2 X^T X of the
- *     layer's inputs); only the upper triangle is read.  Columns whose Hessian
- *     diagonal is zero should be zeroed in W by the caller (they never see input).
+ *   W (device, fp32, [N][K], 16-byte aligned, finite): not modified; a
+ *     non-finite weight gives unspecified (in-range) codes.
+ *   U (device, fp32, [K][K] row-major, 16-byte aligned): the factor from
+ *     logq_gptq_factor (any upper Cholesky factor of a damped inverse Hessian;
+ *     its strictly lower triangle is ignored).
+ *   dead (device, K bytes, may be NULL): inputs marked 1 have their weights
+ *     zeroed before quantisation (they never see input), as logq_gptq_factor
+ *     reports them.
  *   cb (host): the codebook (bits 4 or 8), e.g. from logq_build_codebook with
  *     the range and base of the original W.
  *   codes (device): logq_packed_bytes(N, K, bits) bytes, the packed result.
@@ -248,8 +280,8 @@ size_t logq_gptq_scratch_bytes(int64_t N, int64_t K);
  * LOGQ_ERR_UNSUPPORTED (3-bit codebooks), LOGQ_ERR_WORKSPACE (scratch),
  * LOGQ_ERR_CUDA.
  */
-logq_status logq_gptq(const float* W, int64_t N, int64_t K, const float* U, const logq_codebook* cb,
-                      uint8_t* codes, void* scratch, size_t scratch_bytes, void* stream);
+logq_status logq_gptq(const float* W, int64_t N, int64_t K, const float* U, const uint8_t* dead,
+                      const logq_codebook* cb, uint8_t* codes, void* scratch, size_t scratch_bytes, void* stream);
 
 /* One matrix of logq_linear_grouped. */
 typedef struct logq_linear_item {

@@ -20,9 +20,12 @@ Parity status of each function (what pins it is in ``tests/test_oracle.py``):
   linear               pinned (float64 matmul of the dequantised weights,
                         one-hot and zero inputs)
   energy_wmin          pinned (brute force over all candidate thresholds)
+  gptq_factor          pinned (upper triangular, positive diagonal and U^T U Hd = I,
+                        which fix the Cholesky factor uniquely; a decoupled dead input)
   gptq                 pinned (diagonal Hessian = plain rounding; every compensated
                         value equals the least-squares minimiser given the columns
-                        already quantised, solved directly)
+                        already quantised, solved directly; a dead input = the
+                        reduced problem)
   base_from_range      pinned (closed form: q_max log steps span the range)
 """
 from __future__ import annotations
@@ -146,6 +149,8 @@ def _load():
     lib.oracle_base_from_range.restype = c_dbl
     lib.oracle_gptq.argtypes = [P, c_i64, c_i64, P, c_dbl, ctypes.POINTER(Codebook), P, P]
     lib.oracle_gptq.restype = c_int
+    lib.oracle_gptq_factor.argtypes = [P, c_i64, c_dbl, P]
+    lib.oracle_gptq_factor.restype = c_int
     _lib = lib
     return lib
 
@@ -252,6 +257,17 @@ def linear_sampled(X: np.ndarray, packed: np.ndarray, bits: int, cb: Codebook, t
                                   int(table), _ptr(bs), _ptr(ns), bs.size, _ptr(Y), _ptr(A),
                                   int(nthreads))
     return Y, A
+
+
+def gptq_factor(H, damp: float = 0.01):
+    """U (fp64, upper) with Hd^-1 = U^T U, Hd = H + damp * mean(diag H) * I (a zero
+    diagonal entry of H set to 1 first)."""
+    H = np.ascontiguousarray(H, dtype=np.float64)
+    K = H.shape[0]
+    U = np.empty((K, K), dtype=np.float64)
+    if _load().oracle_gptq_factor(_ptr(H), K, float(damp), _ptr(U)) != 0:
+        raise ValueError("gptq_factor: damped Hessian is not positive definite")
+    return U
 
 
 def gptq(w, H, cb: Codebook, damp: float = 0.01):

@@ -509,23 +509,23 @@ static int chol_lower(double* A, int64_t n)          /* A = L L^T in place (lowe
     return 0;
 }
 
-int oracle_gptq(const float* W, int64_t N, int64_t K, const double* H, double damp,
-                const oracle_codebook* cb, int8_t* q, double* w_at)
+/* The factor GPTQ compensates with: Hd = H + damp * mean(diag H) * I, a zero
+ * diagonal entry of H (an input that never fires) first set to 1; U = the upper
+ * Cholesky factor of Hd^-1 (Hd^-1 = U^T U), fp64 [K][K] row-major, zero below
+ * the diagonal.  Route: Hd = L L^T, Hd^-1 by forward and backward substitution
+ * on the unit columns, then the Cholesky factor of Hd^-1.  Returns 1 if Hd is
+ * not positive definite. */
+int oracle_gptq_factor(const double* H, int64_t K, double damp, double* U)
 {
     double* A = (double*)malloc(sizeof(double) * (size_t)(K * K));
     double* Hinv = (double*)malloc(sizeof(double) * (size_t)(K * K));
-    double* w = (double*)malloc(sizeof(double) * (size_t)(N * K));
     int rc = 1;
     double mean = 0.0;
     for (int64_t j = 0; j < K; ++j) mean += H[j * K + j];
     mean /= (double)K;
     memcpy(A, H, sizeof(double) * (size_t)(K * K));
-    for (int64_t i = 0; i < N * K; ++i) w[i] = (double)W[i];
     for (int64_t j = 0; j < K; ++j) {
-        if (H[j * K + j] == 0.0) {
-            A[j * K + j] = 1.0;
-            for (int64_t r = 0; r < N; ++r) w[r * K + j] = 0.0;
-        }
+        if (H[j * K + j] == 0.0) A[j * K + j] = 1.0;
         A[j * K + j] += damp * mean;
     }
     /* Hd = L L^T; Hd^-1 column by column from L y = e_c, L^T x = y */
@@ -544,6 +544,26 @@ int oracle_gptq(const float* W, int64_t N, int64_t K, const double* H, double da
     }
     /* Hd^-1 = U^T U: U = (lower Cholesky factor of Hd^-1)^T */
     if (chol_lower(Hinv, K)) goto out;
+    for (int64_t j = 0; j < K; ++j)
+        for (int64_t c = 0; c < K; ++c) U[j * K + c] = c >= j ? Hinv[c * K + j] : 0.0;
+    rc = 0;
+out:
+    free(A);
+    free(Hinv);
+    return rc;
+}
+
+int oracle_gptq(const float* W, int64_t N, int64_t K, const double* H, double damp,
+                const oracle_codebook* cb, int8_t* q, double* w_at)
+{
+    double* Uf = (double*)malloc(sizeof(double) * (size_t)(K * K));
+    double* w = (double*)malloc(sizeof(double) * (size_t)(N * K));
+    int rc = 1;
+    for (int64_t i = 0; i < N * K; ++i) w[i] = (double)W[i];
+    for (int64_t j = 0; j < K; ++j)                       /* a dead input's weights are dropped */
+        if (H[j * K + j] == 0.0)
+            for (int64_t r = 0; r < N; ++r) w[r * K + j] = 0.0;
+    if (oracle_gptq_factor(H, K, damp, Uf)) goto out;
     for (int64_t r = 0; r < N; ++r) {
         double* wr = w + r * K;
         for (int64_t j = 0; j < K; ++j) {
@@ -557,15 +577,13 @@ int oracle_gptq(const float* W, int64_t N, int64_t K, const double* H, double da
             q[r * K + j] = qv;
             double deq = (qv < 0 ? -1.0 : 1.0) * (double)cb->level32[m];
             if (m == 0) deq = 0.0;
-            double ujj = Hinv[j * K + j];                  /* U_jj = L^T_jj */
-            double e = (x - deq) / ujj;
-            for (int64_t c = j + 1; c < K; ++c) wr[c] -= e * Hinv[c * K + j];   /* U_jc = L_cj */
+            double e = (x - deq) / Uf[j * K + j];
+            for (int64_t c = j + 1; c < K; ++c) wr[c] -= e * Uf[j * K + c];
         }
     }
     rc = 0;
 out:
-    free(A);
-    free(Hinv);
+    free(Uf);
     free(w);
     return rc;
 }

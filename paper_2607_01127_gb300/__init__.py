@@ -32,6 +32,7 @@ LOGQ_ERR_UNSUPPORTED = 3
 LOGQ_ERR_CUDA = 4
 LOGQ_ERR_WORKSPACE = 5
 LOGQ_ERR_TIMEOUT = 6
+LOGQ_ERR_NOT_PD = 7
 
 LOGQ_F32, LOGQ_BF16, LOGQ_F16 = 0, 1, 2
 LOGQ_SHIFT_EXACT, LOGQ_SHIFT_FLOOR = 0, 1
@@ -39,7 +40,8 @@ LOGQ_SHIFT_EXACT, LOGQ_SHIFT_FLOOR = 0, 1
 EXPORTED = ("logq_build_codebook", "logq_packed_bytes", "logq_workspace_bytes", "logq_quantize",
             "logq_linear", "logq_workspace_status", "logq_status_string", "logq_device_sm_count",
             "logq_quantize_noalloc", "logq_linear_grouped", "logq_energy_scratch_bytes",
-            "logq_quantize_energy", "logq_gptq_scratch_bytes", "logq_gptq")
+            "logq_quantize_energy", "logq_gptq_factor_scratch_bytes", "logq_gptq_factor",
+            "logq_gptq_scratch_bytes", "logq_gptq")
 
 
 class Codebook(ctypes.Structure):
@@ -99,7 +101,11 @@ def _load() -> ctypes.CDLL:
     lib.logq_quantize_energy.restype = c_int
     lib.logq_gptq_scratch_bytes.argtypes = [c_i64, c_i64]
     lib.logq_gptq_scratch_bytes.restype = ctypes.c_size_t
-    lib.logq_gptq.argtypes = [P, c_i64, c_i64, P, ctypes.POINTER(Codebook), P, P, ctypes.c_size_t, P]
+    lib.logq_gptq_factor_scratch_bytes.argtypes = [c_i64]
+    lib.logq_gptq_factor_scratch_bytes.restype = ctypes.c_size_t
+    lib.logq_gptq_factor.argtypes = [P, c_i64, c_dbl, P, P, P, ctypes.c_size_t, P]
+    lib.logq_gptq_factor.restype = c_int
+    lib.logq_gptq.argtypes = [P, c_i64, c_i64, P, P, ctypes.POINTER(Codebook), P, P, ctypes.c_size_t, P]
     lib.logq_gptq.restype = c_int
     lib.logq_linear.argtypes = [P, ctypes.POINTER(Codebook), P, c_int, c_i64, c_i64, c_i64, P,
                                 c_int, P, ctypes.c_size_t, P]
@@ -246,44 +252,43 @@ def logq_quantize_energy(W, bits: int, eps: float = 4e-3, flags: int = LOGQ_SHIF
     return codes[:nbytes], cb, wmin.value
 
 
-def gptq_factor(H, damp: float = 0.01):
-    """Upper Cholesky factor U of the damped inverse Hessian (Hd^-1 = U^T U) that
-    logq_gptq takes, prepared with torch's linear algebra in fp64 on H's device:
-    Hd = H + damp * mean(diag H) * I, a zero diagonal entry set to 1.  Returns
-    (U as fp32, mask of the zero-diagonal columns)."""
+def gptq_factor(H, damp: float = 0.01, U=None, dead=None, scratch=None, stream=None):
+    """U (fp32, upper) with Hd^-1 = U^T U, Hd = H + damp * mean(diag H) * I, and the
+    mask of inputs whose Hessian diagonal is zero, computed by logq_gptq_factor from
+    an fp32 device Hessian H[K, K].  Returns (U, dead)."""
     import torch
-    Hd = H.to(torch.float64).clone()
-    diag = torch.diagonal(Hd)
-    dead = diag == 0
-    mean = diag.mean()
-    idx = torch.nonzero(dead).flatten()
-    Hd[idx, idx] = 1.0
-    Hd += damp * mean * torch.eye(Hd.shape[0], dtype=torch.float64, device=Hd.device)
-    Hinv = torch.cholesky_inverse(torch.linalg.cholesky(Hd))
-    U = torch.linalg.cholesky(Hinv, upper=True)
-    return U.to(torch.float32).contiguous(), dead
+    assert H.dtype == torch.float32 and H.is_cuda and H.dim() == 2 and H.is_contiguous()
+    K = H.shape[0]
+    if U is None:
+        U = torch.empty(K, K, dtype=torch.float32, device=H.device)
+    if dead is None:
+        dead = torch.empty(K, dtype=torch.uint8, device=H.device)
+    if scratch is None:
+        scratch = torch.empty(int(_lib().logq_gptq_factor_scratch_bytes(K)), dtype=torch.uint8, device=H.device)
+    st = _lib().logq_gptq_factor(ctypes.c_void_p(H.data_ptr()), K, float(damp), ctypes.c_void_p(U.data_ptr()),
+                                 ctypes.c_void_p(dead.data_ptr()), ctypes.c_void_p(scratch.data_ptr()),
+                                 scratch.numel(), _stream_ptr(stream))
+    _check(st, "logq_gptq_factor")
+    return U, dead
 
 
 def logq_gptq(W, H, cb: Codebook, damp: float = 0.01, codes=None, scratch=None, stream=None):
-    """GPTQ with the Log_b quantiser: fp32 device weights W[N, K], the layer's
-    Hessian H[K, K] (e.g. 2 X^T X of calibration inputs) and a codebook; returns
-    the packed codes.  The Cholesky factor is prepared by gptq_factor; the column
-    loop and the compensations run in the library's kernels."""
+    """GPTQ with the Log_b quantiser: fp32 device weights W[N, K], the layer's fp32
+    device Hessian H[K, K] (e.g. 2 X^T X of calibration inputs) and a codebook;
+    returns the packed codes.  The factor (logq_gptq_factor), the column loop and
+    the compensations all run in the library's kernels."""
     import torch
     assert W.dtype == torch.float32 and W.is_cuda and W.dim() == 2 and W.is_contiguous()
     N, K = W.shape
-    U, dead = gptq_factor(H, damp)
-    if bool(dead.any()):
-        W = W.clone()
-        W[:, dead] = 0.0
+    U, dead = gptq_factor(H, damp, stream=stream)
     nbytes = logq_packed_bytes(N, K, cb.bits)
     if codes is None:
         codes = torch.empty(max(nbytes, 16), dtype=torch.uint8, device=W.device)
     if scratch is None:
         scratch = torch.empty(int(_lib().logq_gptq_scratch_bytes(N, K)), dtype=torch.uint8, device=W.device)
-    st = _lib().logq_gptq(ctypes.c_void_p(W.data_ptr()), N, K, ctypes.c_void_p(U.data_ptr()), ctypes.byref(cb),
-                          ctypes.c_void_p(codes.data_ptr()), ctypes.c_void_p(scratch.data_ptr()), scratch.numel(),
-                          _stream_ptr(stream))
+    st = _lib().logq_gptq(ctypes.c_void_p(W.data_ptr()), N, K, ctypes.c_void_p(U.data_ptr()),
+                          ctypes.c_void_p(dead.data_ptr()), ctypes.byref(cb), ctypes.c_void_p(codes.data_ptr()),
+                          ctypes.c_void_p(scratch.data_ptr()), scratch.numel(), _stream_ptr(stream))
     _check(st, "logq_gptq")
     if stream is not None:          # the temporaries above belong to the current stream
         stream.synchronize()

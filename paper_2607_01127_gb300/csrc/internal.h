@@ -86,8 +86,12 @@ cudaError_t launch_quantize(const float* W, int64_t N, int64_t K, const QuantPar
                             uint8_t* codes, Workspace* ws, cudaStream_t s);
 cudaError_t launch_gemv(const LinearArgs& a, cudaStream_t s);
 size_t gptq_scratch_bytes(int64_t N, int64_t K);
-cudaError_t launch_gptq(const float* W, int64_t N, int64_t K, const float* U, int bits, const float* thresh,
-                        const float* level, int qmax, uint8_t* codes, void* scratch, cudaStream_t s);
+cudaError_t launch_gptq(const float* W, int64_t N, int64_t K, const float* U, const uint8_t* dead, int bits,
+                        const float* thresh, const float* level, int qmax, uint8_t* codes, void* scratch,
+                        cudaStream_t s);
+size_t gptq_factor_scratch_bytes(int64_t K);
+cudaError_t launch_gptq_factor(const float* H, int64_t K, double damp, float* U, uint8_t* dead, void* scratch,
+                               uint32_t* not_pd, cudaStream_t s);
 cudaError_t launch_gemv_group(const GroupArgs& a, cudaStream_t s);
 cudaError_t launch_prefill(const LinearArgs& a, cudaStream_t s);
 bool gemv_supports(int bits, int64_t B);

@@ -252,14 +252,33 @@ logq_status logq_quantize_energy(const float* W, int64_t N, int64_t K, int bits,
     return LOGQ_OK;
 }
 
+size_t logq_gptq_factor_scratch_bytes(int64_t K)
+{
+    if (K <= 0 || (K % 128) != 0 || K > 65536) return 0;
+    return gptq_factor_scratch_bytes(K);
+}
+
+logq_status logq_gptq_factor(const float* H, int64_t K, double damp, float* U, uint8_t* dead, void* scratch,
+                             size_t scratch_bytes, void* stream)
+{
+    if (!H || !U || !aligned16(H) || !aligned16(U)) return LOGQ_ERR_INVALID_ARG;
+    if (K <= 0 || (K % 128) != 0 || K > 65536) return LOGQ_ERR_INVALID_ARG;
+    if (!(damp >= 0.0) || !isfinite(damp)) return LOGQ_ERR_INVALID_ARG;
+    if (!scratch || !aligned16(scratch) || scratch_bytes < gptq_factor_scratch_bytes(K)) return LOGQ_ERR_WORKSPACE;
+    uint32_t not_pd = 0;
+    const cudaError_t e = launch_gptq_factor(H, K, damp, U, dead, scratch, &not_pd, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_status(e);
+    return not_pd ? LOGQ_ERR_NOT_PD : LOGQ_OK;
+}
+
 size_t logq_gptq_scratch_bytes(int64_t N, int64_t K)
 {
     if (N <= 0 || K <= 0 || (K % 128) != 0) return 0;
     return gptq_scratch_bytes(N, K);
 }
 
-logq_status logq_gptq(const float* W, int64_t N, int64_t K, const float* U, const logq_codebook* cb,
-                      uint8_t* codes, void* scratch, size_t scratch_bytes, void* stream)
+logq_status logq_gptq(const float* W, int64_t N, int64_t K, const float* U, const uint8_t* dead,
+                      const logq_codebook* cb, uint8_t* codes, void* scratch, size_t scratch_bytes, void* stream)
 {
     if (!W || !U || !cb || !codes) return LOGQ_ERR_INVALID_ARG;
     if (!aligned16(W) || !aligned16(U) || !aligned16(codes)) return LOGQ_ERR_INVALID_ARG;
@@ -268,7 +287,7 @@ logq_status logq_gptq(const float* W, int64_t N, int64_t K, const float* U, cons
     if (N > (int64_t(1) << 40) / K) return LOGQ_ERR_INVALID_ARG;
     if (cb->bits != 4 && cb->bits != 8) return LOGQ_ERR_UNSUPPORTED;
     if (!scratch || !aligned16(scratch) || scratch_bytes < gptq_scratch_bytes(N, K)) return LOGQ_ERR_WORKSPACE;
-    const cudaError_t e = launch_gptq(W, N, K, U, cb->bits, cb->thresh, cb->level, cb->qmax, codes, scratch,
+    const cudaError_t e = launch_gptq(W, N, K, U, dead, cb->bits, cb->thresh, cb->level, cb->qmax, codes, scratch,
                                       static_cast<cudaStream_t>(stream));
     return cuda_status(e);
 }
@@ -387,6 +406,7 @@ const char* logq_status_string(logq_status status)
     case LOGQ_ERR_CUDA: return "CUDA runtime error";
     case LOGQ_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
     case LOGQ_ERR_TIMEOUT: return "device pipeline wait exceeded its bound";
+    case LOGQ_ERR_NOT_PD: return "damped Hessian is not positive definite";
     }
     return "unknown status";
 }

@@ -171,7 +171,7 @@ def test_gptq_rejects_before_launch(logq):
     assert L.logq_gptq_scratch_bytes(64, 100) == 0
 
     def call(W=W, U=U, cb=cb4, C=C, sc=sc, scb=scb, N=64, K=256):
-        return L.logq_gptq(W, N, K, U, ctypes.byref(cb), C, sc, scb, None)
+        return L.logq_gptq(W, N, K, U, None, ctypes.byref(cb), C, sc, scb, None)
 
     assert call(W=None) == logq.LOGQ_ERR_INVALID_ARG
     assert call(U=_fake(0x20004)) == logq.LOGQ_ERR_INVALID_ARG
@@ -179,6 +179,29 @@ def test_gptq_rejects_before_launch(logq):
     assert call(cb=cb3) == logq.LOGQ_ERR_UNSUPPORTED
     assert call(sc=None) == logq.LOGQ_ERR_WORKSPACE
     assert call(scb=scb - 16) == logq.LOGQ_ERR_WORKSPACE
+
+
+def test_gptq_factor_rejects_before_launch(logq):
+    """logq_gptq_factor validates sizes, damping and scratch before anything is enqueued."""
+    L = logq.lib
+    H, U, sc = _fake(0x10000), _fake(0x20000), _fake(0x40000)
+    scb = L.logq_gptq_factor_scratch_bytes(256)
+    assert scb == 256 + (256 * 256 + 256 * 256 // 4) * 4
+    assert L.logq_gptq_factor_scratch_bytes(100) == 0
+    assert L.logq_gptq_factor_scratch_bytes(0) == 0
+
+    def call(H=H, K=256, damp=0.01, U=U, sc=sc, scb=scb):
+        return L.logq_gptq_factor(H, K, damp, U, None, sc, scb, None)
+
+    assert call(H=None) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(U=_fake(0x20004)) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(K=100) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(K=-128) == logq.LOGQ_ERR_INVALID_ARG
+    for damp in (-0.01, float("nan"), float("inf")):
+        assert call(damp=damp) == logq.LOGQ_ERR_INVALID_ARG
+    assert call(sc=None) == logq.LOGQ_ERR_WORKSPACE
+    assert call(scb=scb - 4) == logq.LOGQ_ERR_WORKSPACE
+    assert logq.status_string(logq.LOGQ_ERR_NOT_PD) == "damped Hessian is not positive definite"
 
 
 def test_linear_rejects_before_launch(logq):

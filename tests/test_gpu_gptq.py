@@ -1,5 +1,6 @@
-"""GPTQ with the Log_b quantiser on the device against the fp64 oracle: a
-diagonal Hessian reduces it to plain rounding (codes bit-exact against
+"""GPTQ with the Log_b quantiser on the device against the fp64 oracle: the
+factor U (fp32 on the device) against the oracle's within fp32 accuracy; a
+diagonal Hessian reduces GPTQ to plain rounding (codes bit-exact against
 logq_quantize); on correlated synthetic inputs the codes agree with the
 oracle's except where fp32 and fp64 compensations put a weight on different
 sides of a boundary (a small, counted fraction), and the layer loss
@@ -34,13 +35,39 @@ def loss(w, q, cb, H):
     return float(np.einsum("ij,jk,ik->", d, H, d))
 
 
+@pytest.mark.parametrize("K", [128, 384, 640, 1152])
+def test_gptq_factor_matches_oracle(logq, K):
+    """U from the device (fp32 Cholesky of the reversed Hessian, blocked triangular
+    inverse; 2, 6, 10 and 18 blocks of 64, so the inverse's doubling meets
+    complete and shortened pairs) against the oracle's fp64 factor, with a
+    dead input."""
+    H = hessian(K, 50 + K)
+    H[3, :] = H[:, 3] = 0.0
+    Hf = H.astype(np.float32)
+    U, dead = logq.gptq_factor(torch.from_numpy(Hf).cuda(), 0.01)
+    U = U.double().cpu().numpy()
+    Uo = oracle.gptq_factor(Hf.astype(np.float64), 0.01)
+    assert np.all(np.tril(U, -1) == 0.0)
+    err = float(np.max(np.abs(U - Uo)) / np.max(np.abs(Uo)))
+    assert err < 2e-4, err
+    np.testing.assert_array_equal(dead.cpu().numpy(), (np.diag(Hf) == 0).astype(np.uint8))
+    assert np.all(U[3, 4:] == 0.0) and np.all(U[:3, 3] == 0.0)
+
+
+def test_gptq_factor_not_positive_definite(logq):
+    H = -torch.eye(256, device="cuda")
+    with pytest.raises(logq.LogqError) as ei:
+        logq.gptq_factor(H, 0.01)
+    assert ei.value.status == logq.LOGQ_ERR_NOT_PD
+
+
 @pytest.mark.parametrize("bits,base", [(4, 1.5), (8, 1.05)])
 def test_gptq_diagonal_hessian_is_plain_rounding(logq, bits, base):
     N, K = 96, 384
     w = workloads.weights_np(N, K, seed=3, outliers=True)
     W = torch.from_numpy(w).cuda()
     cb = logq.logq_build_codebook(bits, base, float(np.abs(w).max()))
-    H = torch.diag(torch.rand(K, dtype=torch.float64, generator=torch.Generator().manual_seed(1)) + 0.5).cuda()
+    H = torch.diag(torch.rand(K, dtype=torch.float32, generator=torch.Generator().manual_seed(1)) + 0.5).cuda()
     codes = logq.logq_gptq(W, H, cb)
     ref, _ = logq.logq_quantize(W, bits, base, float(np.abs(w).max()))
     assert torch.equal(codes, ref)
@@ -52,7 +79,7 @@ def test_gptq_matches_oracle(logq, bits, base, N, K):
     w = workloads.weights_np(N, K, seed=N + K + bits, outliers=True)
     H = hessian(K, K + bits)
     cb = logq.logq_build_codebook(bits, base, float(np.abs(w).max()))
-    codes = logq.logq_gptq(torch.from_numpy(w).cuda(), torch.from_numpy(H).cuda(), cb)
+    codes = logq.logq_gptq(torch.from_numpy(w).cuda(), torch.from_numpy(H).float().cuda(), cb)
     q_dev = oracle.unpack(codes.cpu().numpy().reshape(N, -1), N, K, bits)
     ocb = oracle.build_codebook(bits, base, float(np.abs(w).max()))
     q_ref, _ = oracle.gptq(w, H, ocb)
@@ -70,7 +97,7 @@ def test_gptq_repeatable_and_dead_columns(logq):
     H = hessian(K, 9)
     H[:, 5] = H[5, :] = 0.0                           # an input that never fires
     cb = logq.logq_build_codebook(4, 1.4, float(np.abs(w).max()))
-    W, Ht = torch.from_numpy(w).cuda(), torch.from_numpy(H).cuda()
+    W, Ht = torch.from_numpy(w).cuda(), torch.from_numpy(H).float().cuda()
     c1, c2 = logq.logq_gptq(W, Ht, cb), logq.logq_gptq(W, Ht, cb)
     assert torch.equal(c1, c2)
     q = oracle.unpack(c1.cpu().numpy().reshape(N, -1), N, K, 4)
@@ -97,7 +124,7 @@ def test_gptq_full_size_q_8b(logq):
     g = torch.Generator(device="cuda").manual_seed(6)
     X = torch.randn(3 * K, K, device="cuda", generator=g, dtype=torch.float64)
     X[:, 1:] += 0.5 * X[:, :-1].clone()
-    H = X.T @ X
+    H = (X.T @ X).float()
     del X
     # the paper's codebook: range and base from the weights (Eqs. (3)-(5), eps = 4e-3);
     # logq_quantize_energy's own codes are plain rounding with it
@@ -110,7 +137,7 @@ def test_gptq_full_size_q_8b(logq):
         return lv[q].double()
     def L(c):
         d = W.double() - deq(c)
-        return float(((d @ H) * d).sum())
+        return float(((d @ H.double()) * d).sum())
     l_gptq, l_rtn = L(codes), L(rtn)
     print(f"layer loss: GPTQ {l_gptq:.6g}, rounding {l_rtn:.6g}")
     assert l_gptq < l_rtn

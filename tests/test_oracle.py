@@ -374,3 +374,40 @@ def test_gptq_lowers_the_layer_loss():
     loss = lambda qq: float(np.trace((w - oracle.dequant(qq, cb, oracle.TABLE_F32)) @ H @
                                      (w - oracle.dequant(qq, cb, oracle.TABLE_F32)).T))
     assert loss(q) < 0.9 * loss(oracle.quantize_thresh(w, cb))
+
+
+@pytest.mark.parametrize("bits", [4, 8])
+def test_gptq_dead_input_is_the_reduced_problem(bits):
+    """An input that never fires (zero Hessian row and column) is dropped: its
+    weights code 0, and the other columns come out as GPTQ of the matrix without
+    that column (damping rescaled so that damp * mean(diag) is the same)."""
+    N, K, d = 6, 20, 7
+    w = workloads.weights_np(N, K, 21)
+    cb = oracle.build_codebook(bits, 1.4 if bits == 4 else 1.05, float(np.abs(w).max()))
+    H = _hessian(K, 22)
+    H[d, :] = H[:, d] = 0.0
+    q, w_at = oracle.gptq(w, H, cb, 0.01)
+    keep = [k for k in range(K) if k != d]
+    q_r, w_r = oracle.gptq(np.ascontiguousarray(w[:, keep]), H[np.ix_(keep, keep)], cb, 0.01 * (K - 1) / K)
+    assert np.all(q[:, d] == 0) and np.all(w_at[:, d] == 0.0)
+    np.testing.assert_array_equal(q[:, keep], q_r)
+    np.testing.assert_allclose(w_at[:, keep], w_r, rtol=1e-12, atol=1e-15)
+
+
+@pytest.mark.parametrize("K", [1, 5, 64])
+def test_gptq_factor_is_the_cholesky_factor_of_the_inverse(K):
+    """U is upper triangular with a positive diagonal and U^T U Hd = I: the
+    Cholesky factor of Hd^-1 is the only such matrix."""
+    H = _hessian(K, 30 + K)
+    if K > 2:
+        H[2, :] = H[:, 2] = 0.0                       # a dead input: decoupled, diagonal 1 + damping
+    damp = 0.01
+    U = oracle.gptq_factor(H, damp)
+    mean = np.mean(np.diag(H))
+    Hd = H + damp * mean * np.eye(K)
+    if K > 2:
+        Hd[2, 2] = 1.0 + damp * mean
+        assert U[2, 2] == pytest.approx(1.0 / np.sqrt(Hd[2, 2]), rel=1e-14)
+        assert np.all(U[2, 3:] == 0.0) and np.all(U[:2, 2] == 0.0)
+    assert np.all(np.tril(U, -1) == 0.0) and np.all(np.diag(U) > 0)
+    np.testing.assert_allclose(U.T @ U @ Hd, np.eye(K), atol=1e-9)
