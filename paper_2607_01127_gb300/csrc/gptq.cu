@@ -212,44 +212,42 @@ __global__ void gptq_prep_kernel(const float* __restrict__ H, int64_t K, double 
 
 // Cholesky of the 64 x 64 diagonal block at (k0, k0) (lower triangle read),
 // then the inverse of its factor, written back in its place with zeros above
-// the diagonal.  One CTA.
+// the diagonal.  One CTA of 256 threads: a 16 x 16 layout for the updates, four
+// threads per column of the inverse.
 __global__ void __launch_bounds__(256) gptq_potrf_kernel(float* __restrict__ A, int64_t K, int64_t k0,
                                                          FactorState* st)
 {
     __shared__ float a[kNb][kNb + 1];
     __shared__ float inv[kNb][kNb + 1];
-    const int tid = threadIdx.x;
+    const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
     for (int i = tid; i < kNb * kNb; i += 256) {
         const int r = i / kNb, c = i % kNb;
         a[r][c] = c <= r ? A[(k0 + r) * K + k0 + c] : 0.f;
     }
     __syncthreads();
     for (int j = 0; j < kNb; ++j) {
-        if (tid == 0) {
-            const float d = a[j][j];
-            if (!(d > 0.f) || !isfinite(d)) st->not_pd = 1;
-            a[j][j] = sqrtf(d);
-        }
+        const float p = a[j][j];
+        const float d = sqrtf(p);
+        if (tid == 0 && (!(p > 0.f) || !isfinite(p))) st->not_pd = 1;
+        if (tid > j && tid < kNb) a[tid][j] = a[tid][j] / d;
         __syncthreads();
-        if (tid > j && tid < kNb) a[tid][j] = a[tid][j] / a[j][j];
-        __syncthreads();
-        const int n = kNb - 1 - j;
-        for (int idx = tid; idx < n * n; idx += 256) {
-            const int i = j + 1 + idx / n, k = j + 1 + idx % n;
-            if (k <= i) a[i][k] -= a[i][j] * a[k][j];
+        if (tid == 0) a[j][j] = d;
+        for (int i = j + 1 + ty; i < kNb; i += 16) {
+            const float lij = a[i][j];
+            for (int k = j + 1 + tx; k <= i; k += 16) a[i][k] -= lij * a[k][j];
         }
         __syncthreads();
     }
-    if (tid < kNb) {                         // column tid of the inverse, forward substitution
-        const int c = tid;
+    {   // column c of the inverse by forward substitution, each sum split over four lanes
+        const int c = tid / 4, q = tid % 4;
         for (int i = 0; i < kNb; ++i) {
-            if (i < c) {
-                inv[i][c] = 0.f;
-                continue;
-            }
-            float s = i == c ? 1.f : 0.f;
-            for (int k = c; k < i; ++k) s -= a[i][k] * inv[k][c];
-            inv[i][c] = s / a[i][i];
+            float part = 0.f;
+            if (i > c)
+                for (int k = c + q; k < i; k += 4) part = fmaf(a[i][k], inv[k][c], part);
+            part += __shfl_xor_sync(0xffffffffu, part, 1);
+            part += __shfl_xor_sync(0xffffffffu, part, 2);
+            if (q == 0) inv[i][c] = i < c ? 0.f : ((i == c ? 1.f : 0.f) - part) / a[i][i];
+            __syncwarp();
         }
     }
     __syncthreads();
