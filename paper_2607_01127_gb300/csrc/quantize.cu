@@ -4,12 +4,21 @@
 // The quantiser assigns m = #{ j : |w| >= thresh[j] } against the fp32
 // decision boundaries of the codebook (rounded up from fp64), which for fp32
 // weights equals round(log_b|w| + s) clamped to [0, q_max].
+#include <math.h>
 #include <stdint.h>
+#include <string.h>
 
 #include "internal.h"
 
 namespace logq {
 namespace {
+
+struct QuantEst {
+    uint32_t t2[8];     // 2 x the boundaries' bit patterns; 0xffffffff after the last
+    uint64_t C;         // fixed-point offset of the level estimate (two's complement)
+    uint32_t K;         // fixed-point slope
+    uint32_t _pad;
+};
 
 __device__ __forceinline__ float4 ld_stream(const float4* p)
 {
@@ -133,6 +142,49 @@ __global__ void __launch_bounds__(256) quantize4_kernel(const float4* __restrict
     }
 }
 
+// 4-bit with the level estimated from the weight's bit pattern.  The bit
+// pattern u of a positive normal float, read as an integer, is a piecewise-linear
+// log2: u / 2^23 - 127 = e + f, below log2 by at most 0.0861.  With the
+// boundaries geometric (ratio b = 2^lambda, lambda >= 0.12), the fixed-point
+// value floor(((2u - U0) K + C) / 2^32), a little below the level count the
+// real log2 would give, is the true count m or m - 1; one comparison with the
+// boundary m_est decides: m = m_est + (|w| >= thresh[m_est]).  The decision is
+// the boundary comparison itself, so the codes equal quantize4_kernel's.  The
+// host sets K, C and the guards (first boundary normal, lambda in [0.12, 3]).
+template <bool CHECK>
+__global__ void __launch_bounds__(256) quantize4e_kernel(const float4* __restrict__ W, int64_t nwords,
+                                                         const __grid_constant__ QuantEst q,
+                                                         uint32_t* __restrict__ out, Workspace* ws)
+{
+    __shared__ uint32_t t2[8];
+    if (threadIdx.x < 8) t2[threadIdx.x] = q.t2[threadIdx.x];
+    __syncthreads();
+    uint32_t umax = 0;                       // largest 2|w| bit pattern seen (non-finite check)
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nwords; i += stride) {
+        const float4 a = ld_stream(W + 2 * i);
+        const float4 b = ld_stream(W + 2 * i + 1);
+        const float v[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+        uint32_t mword = 0, sword = 0;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const uint32_t bits = __float_as_uint(v[e]);
+            const uint32_t u2 = bits << 1;   // 2|w|: the sign bit drops out
+            if (CHECK) umax = max(umax, u2);
+            const uint64_t p = (uint64_t)u2 * q.K + q.C;
+            const int mh = __vimin_s32_relu((int)(uint32_t)(p >> 32), 7);
+            mword |= ((uint32_t)mh + (u2 >= t2[mh] ? 1u : 0u)) << (4 * e);
+            sword |= (bits >> 31) << (4 * e + 3);
+        }
+        // a sign bit only on nibbles whose magnitude is not 0 (m + 7 carries into bit 3)
+        out[i] = mword | (sword & (mword + 0x77777777u) & 0x88888888u);
+    }
+    if (CHECK) {
+        const uint32_t bad = __reduce_or_sync(0xffffffffu, umax >= 0xff000000u ? 1u : 0u);
+        if (bad && (threadIdx.x & 31) == 0) atomicOr(&ws->nonfinite, 1u);
+    }
+}
+
 // 3-bit: each thread packs one group of 32 weights into 12 bytes.
 __global__ void __launch_bounds__(256) quantize3_kernel(const float4* __restrict__ W, int64_t ngroups,
                                                         QuantParams p, uint32_t* __restrict__ out,
@@ -225,6 +277,35 @@ __global__ void __launch_bounds__(256) quantize8_kernel(const float4* __restrict
     }
 }
 
+// Fixed-point slope and offset of quantize4e_kernel's level estimate, from the
+// 4-bit boundaries; false when the guards fail (the boundary search is used).
+//   lambda = log2 of the boundary ratio, from the first and last boundary;
+//   estimate(u2) = floor((u2 K + C) / 2^32) with K = round(2^8 / lambda) and
+//   C = round(-(log2 t_0 + 127) 2^24 K + (1 - 0.05) 2^32), i.e. the level count
+//   from the linear log2 of the bit pattern, biased down by 0.05 of a level so
+//   that the rounding of K, C and of the boundaries never lifts it above the
+//   true count; the linear log2 lies below log2 by at most 0.0861, i.e.
+//   0.0861 / lambda <= 0.72 levels for lambda >= 0.12.
+bool estimate_params(const QuantParams& p, QuantEst& q)
+{
+    if (p.bits != 4 || p.qmax != 7) return false;
+    const double t0 = p.thresh[0], t6 = p.thresh[6];
+    if (!(t0 >= 1.1754943508222875e-38) || !(t6 > t0) || !isfinite(t6)) return false;
+    const double l0 = log2(t0);
+    const double lambda = (log2(t6) - l0) / 6.0;
+    if (!(lambda >= 0.12) || !(lambda <= 3.0)) return false;
+    const double k = nearbyint(256.0 / lambda);
+    q.K = (uint32_t)k;
+    q.C = (uint64_t)(int64_t)nearbyint(-(l0 + 127.0) * 16777216.0 * k + 0.95 * 4294967296.0);
+    for (int j = 0; j < 7; ++j) {
+        uint32_t b;
+        memcpy(&b, &p.thresh[j], 4);
+        q.t2[j] = 2u * b;
+    }
+    q.t2[7] = 0xffffffffu;
+    return true;
+}
+
 int grid_for(int64_t items, int threads)
 {
     const int sms = sm_count() > 0 ? sm_count() : 148;
@@ -252,8 +333,18 @@ cudaError_t launch_quantize(const float* W, int64_t N, int64_t K, const QuantPar
             reinterpret_cast<const float4*>(W), n16, p, reinterpret_cast<uint4*>(codes), ws);
     } else if (p.bits == 4) {
         const int64_t nwords = total / 8;
-        quantize4_kernel<<<grid_for(nwords, 256), 256, 0, s>>>(
-            reinterpret_cast<const float4*>(W), nwords, p, reinterpret_cast<uint32_t*>(codes), ws);
+        QuantEst q;
+        if (estimate_params(p, q)) {
+            if (p.check_nonfinite)
+                quantize4e_kernel<true><<<grid_for(nwords, 256), 256, 0, s>>>(
+                    reinterpret_cast<const float4*>(W), nwords, q, reinterpret_cast<uint32_t*>(codes), ws);
+            else
+                quantize4e_kernel<false><<<grid_for(nwords, 256), 256, 0, s>>>(
+                    reinterpret_cast<const float4*>(W), nwords, q, reinterpret_cast<uint32_t*>(codes), ws);
+        } else {
+            quantize4_kernel<<<grid_for(nwords, 256), 256, 0, s>>>(
+                reinterpret_cast<const float4*>(W), nwords, p, reinterpret_cast<uint32_t*>(codes), ws);
+        }
     } else {
         const int64_t ngroups = total / 32;
         quantize3_kernel<<<grid_for(ngroups, 256), 256, 0, s>>>(

@@ -100,3 +100,25 @@ def test_quantize_repeatable(logq):
     a, _ = logq.logq_quantize(W, 4, 1.7)
     b, _ = logq.logq_quantize(W, 4, 1.7)
     assert torch.equal(a, b)
+
+
+@pytest.mark.parametrize("base", [1.05, 1.087, 1.1, 1.5, 3.0, 7.9, 9.0])
+@pytest.mark.parametrize("mode", [0, 1])
+def test_quantize4_every_boundary_and_neighbours(logq, base, mode):
+    """4-bit codes of every fp32 boundary, its two fp32 neighbours on each side, both
+    signs, subnormals, zeros and values far outside the range: bit-exact.  Bases from
+    1.05 to 9 cover the boundary search and the estimate-and-correct kernel (used for
+    boundary ratios 2^0.12 to 2^3) on both sides of its guards."""
+    rng_ = 0.75
+    ocb = oracle.build_codebook(4, base, rng_, mode)
+    t = np.asarray(ocb.taus32_up, np.float32)
+    near = np.concatenate([t, np.nextafter(t, np.float32(0)), np.nextafter(t, np.float32(np.inf)),
+                           np.nextafter(np.nextafter(t, np.float32(0)), np.float32(0)),
+                           np.nextafter(np.nextafter(t, np.float32(np.inf)), np.float32(np.inf))])
+    extra = np.float32([0.0, -0.0, 1e-45, -1e-45, 1e-39, 1.1754942e-38, 1.1754944e-38, 1e-20, 0.5, 0.75,
+                        0.7500001, 3.0, 1e30, 3.4e38, -3.4e38])
+    rnd = (np.random.default_rng(int(base * 1000) + mode).standard_normal(128 * 64) * 0.3).astype(np.float32)
+    w = np.concatenate([near, -near, extra, rnd]).astype(np.float32)
+    w = np.concatenate([w, np.zeros((-w.size) % 128, np.float32)]).reshape(-1, 128)
+    codes, cb = logq.logq_quantize(torch.from_numpy(w).cuda(), 4, base, rng_, mode)
+    assert check_codes(codes.cpu().numpy(), w, ocb, 4) == 0
