@@ -20,6 +20,14 @@ struct QuantEst {
     uint32_t _pad;
 };
 
+struct QuantEst8 {
+    uint32_t t2[128];   // 2 x the 127 boundaries' bit patterns; 0xffffffff at 127
+    uint32_t corr[64];  // log2(1 + f) - f (lower bound over each 1/64 of f), in units of 2^-24
+    uint64_t C;         // fixed-point offset (two's complement), units of 2^-40 of a level
+    uint32_t K;         // fixed-point slope
+    uint32_t _pad;
+};
+
 __device__ __forceinline__ float4 ld_stream(const float4* p)
 {
     float4 v;
@@ -185,6 +193,53 @@ __global__ void __launch_bounds__(256) quantize4e_kernel(const float4* __restric
     }
 }
 
+// 8-bit with the level estimated as in quantize4e_kernel, the linear log2 of
+// the bit pattern corrected by a 64-entry table over the top 6 mantissa bits
+// (a lower bound of log2(1 + f) - f on each interval, so the estimate stays
+// below log2 by at most 0.0069) and a 40-bit fixed point (127 levels): for
+// boundary ratios 2^lambda with lambda >= 0.01 the estimate is the true count
+// m or m - 1 and one comparison with the fp32 boundary decides.
+template <bool CHECK>
+__global__ void __launch_bounds__(256) quantize8e_kernel(const float4* __restrict__ W, int64_t n16,
+                                                         const __grid_constant__ QuantEst8 q,
+                                                         uint4* __restrict__ out, Workspace* ws)
+{
+    __shared__ uint32_t t2[128];
+    __shared__ uint32_t corr[64];
+    if (threadIdx.x < 128) t2[threadIdx.x] = q.t2[threadIdx.x];
+    if (threadIdx.x < 64) corr[threadIdx.x] = q.corr[threadIdx.x];
+    __syncthreads();
+    uint32_t umax = 0;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n16; i += stride) {
+        float4 v4[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) v4[j] = ld_stream(W + 4 * i + j);
+        uint32_t word[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const float v[4] = {v4[j].x, v4[j].y, v4[j].z, v4[j].w};
+            uint32_t mword = 0, sword = 0;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const uint32_t bits = __float_as_uint(v[e]);
+                const uint32_t u2 = bits << 1;
+                if (CHECK) umax = max(umax, u2);
+                const uint64_t p = (uint64_t)(u2 + corr[(u2 >> 18) & 63]) * q.K + q.C;
+                const int mh = __vimin_s32_relu((int)(uint32_t)(p >> 32) >> 8, 127);
+                mword |= ((uint32_t)mh + (u2 >= t2[mh] ? 1u : 0u)) << (8 * e);
+                sword |= (bits >> 31) << (8 * e + 7);
+            }
+            word[j] = mword | (sword & (mword + 0x7f7f7f7fu) & 0x80808080u);
+        }
+        out[i] = make_uint4(word[0], word[1], word[2], word[3]);
+    }
+    if (CHECK) {
+        const uint32_t bad = __reduce_or_sync(0xffffffffu, umax >= 0xff000000u ? 1u : 0u);
+        if (bad && (threadIdx.x & 31) == 0) atomicOr(&ws->nonfinite, 1u);
+    }
+}
+
 // 3-bit: each thread packs one group of 32 weights into 12 bytes.
 __global__ void __launch_bounds__(256) quantize3_kernel(const float4* __restrict__ W, int64_t ngroups,
                                                         QuantParams p, uint32_t* __restrict__ out,
@@ -306,6 +361,36 @@ bool estimate_params(const QuantParams& p, QuantEst& q)
     return true;
 }
 
+// quantize8e_kernel's parameters (lambda and the table as above, K = round(2^16 /
+// lambda), C = round(-(log2 t_0 + 127) 2^24 K + 0.95 2^40)); false when the guards
+// fail: first boundary below 2^-120 (subnormal weights plus the table's
+// correction must stay below it) or lambda outside [0.01, 4].
+bool estimate_params8(const QuantParams& p, QuantEst8& q)
+{
+    if (p.bits != 8 || p.qmax != 127) return false;
+    const double t0 = p.thresh[0], tl = p.thresh[126];
+    if (!(t0 >= 7.52316384526264e-37) || !(tl > t0) || !isfinite(tl)) return false;   // 2^-120
+    const double l0 = log2(t0);
+    const double lambda = (log2(tl) - l0) / 126.0;
+    if (!(lambda >= 0.01) || !(lambda <= 4.0)) return false;
+    const double k = nearbyint(65536.0 / lambda);
+    q.K = (uint32_t)k;
+    q.C = (uint64_t)(int64_t)nearbyint(-(l0 + 127.0) * 16777216.0 * k + 0.95 * 1099511627776.0);
+    for (int j = 0; j < 127; ++j) {
+        uint32_t b;
+        memcpy(&b, &p.thresh[j], 4);
+        q.t2[j] = 2u * b;
+    }
+    q.t2[127] = 0xffffffffu;
+    for (int i = 0; i < 64; ++i) {
+        const double f0 = i / 64.0, f1 = (i + 1) / 64.0;
+        const double g0 = log2(1.0 + f0) - f0, g1 = log2(1.0 + f1) - f1;   // concave: minimum at an end
+        q.corr[i] = (uint32_t)floor(16777216.0 * (g0 < g1 ? g0 : g1));
+    }
+    q._pad = 0;
+    return true;
+}
+
 int grid_for(int64_t items, int threads)
 {
     const int sms = sm_count() > 0 ? sm_count() : 148;
@@ -329,8 +414,18 @@ cudaError_t launch_quantize(const float* W, int64_t N, int64_t K, const QuantPar
     const int64_t total = N * K;
     if (p.bits == 8) {
         const int64_t n16 = total / 16;
-        quantize8_kernel<<<grid_for(n16, 256), 256, 0, s>>>(
-            reinterpret_cast<const float4*>(W), n16, p, reinterpret_cast<uint4*>(codes), ws);
+        QuantEst8 q;
+        if (estimate_params8(p, q)) {
+            if (p.check_nonfinite)
+                quantize8e_kernel<true><<<grid_for(n16, 256), 256, 0, s>>>(
+                    reinterpret_cast<const float4*>(W), n16, q, reinterpret_cast<uint4*>(codes), ws);
+            else
+                quantize8e_kernel<false><<<grid_for(n16, 256), 256, 0, s>>>(
+                    reinterpret_cast<const float4*>(W), n16, q, reinterpret_cast<uint4*>(codes), ws);
+        } else {
+            quantize8_kernel<<<grid_for(n16, 256), 256, 0, s>>>(
+                reinterpret_cast<const float4*>(W), n16, p, reinterpret_cast<uint4*>(codes), ws);
+        }
     } else if (p.bits == 4) {
         const int64_t nwords = total / 8;
         QuantEst q;

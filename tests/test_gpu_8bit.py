@@ -143,3 +143,24 @@ def test_prefill8(logq, N, K, B, ydt):
     check_linear(Y.double().cpu().numpy(), Yr, A, "f32" if ydt is None else "bf16")
     st, _ = logq.logq_workspace_status(ws)
     assert st == logq.LOGQ_OK
+
+
+@pytest.mark.parametrize("base", [1.005, 1.0075, 1.02, 1.05, 1.1, 1.5, 2.0])
+@pytest.mark.parametrize("mode", [0, 1])
+def test_quantize8_every_boundary_and_neighbours(logq, base, mode):
+    """8-bit codes of all 127 fp32 boundaries, their fp32 neighbours, both signs,
+    subnormals, zeros and values far outside the range: bit-exact.  The bases cover
+    the estimate-and-correct kernel (boundary ratios 2^0.01 .. 2^4, first boundary at
+    least 2^-120) and the boundary search on both sides of its guards."""
+    rng_ = 0.75
+    ocb = oracle.build_codebook(8, base, rng_, mode)
+    t = np.asarray(ocb.taus32_up, np.float32)
+    t = t[t > 0]
+    near = np.concatenate([t, np.nextafter(t, np.float32(0)), np.nextafter(t, np.float32(np.inf))])
+    extra = np.float32([0.0, -0.0, 1e-45, -1e-45, 1e-39, 1.1754942e-38, 1e-30, 0.5, 0.75, 0.7500001,
+                        3.0, 1e30, 3.4e38, -3.4e38])
+    rnd = (np.random.default_rng(int(base * 1e4) + mode).standard_normal(128 * 32) * 0.2).astype(np.float32)
+    w = np.concatenate([near, -near, extra, rnd]).astype(np.float32)
+    w = np.concatenate([w, np.zeros((-w.size) % 128, np.float32)]).reshape(-1, 128)
+    codes, cb = logq.logq_quantize(torch.from_numpy(w).cuda(), 8, base, rng_, mode)
+    assert check_codes(codes.cpu().numpy(), w, ocb, 8) == 0
