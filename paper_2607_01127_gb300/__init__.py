@@ -258,6 +258,7 @@ def gptq_factor(H, damp: float = 0.01, U=None, dead=None, scratch=None, stream=N
     an fp32 device Hessian H[K, K].  Returns (U, dead)."""
     import torch
     assert H.dtype == torch.float32 and H.is_cuda and H.dim() == 2 and H.is_contiguous()
+    assert H.shape[0] == H.shape[1], "H must be square"
     K = H.shape[0]
     if U is None:
         U = torch.empty(K, K, dtype=torch.float32, device=H.device)
@@ -280,6 +281,7 @@ def logq_gptq(W, H, cb: Codebook, damp: float = 0.01, codes=None, scratch=None, 
     import torch
     assert W.dtype == torch.float32 and W.is_cuda and W.dim() == 2 and W.is_contiguous()
     N, K = W.shape
+    assert tuple(H.shape) == (K, K), "H must be K x K for W of K columns"
     U, dead = gptq_factor(H, damp, stream=stream)
     nbytes = logq_packed_bytes(N, K, cb.bits)
     if codes is None:
