@@ -9,12 +9,15 @@
  *   q_max = 2^(n-1) - 1 for an n-bit code; Eq. (4) aligns w_max with q_max.
  *
  * Inference multiplies activations with the dequantised weights through a
- * lookup table (Sec. 3.3).  This library provides the three steps of that
- * path as device kernels behind plain C calls:
+ * lookup table (Sec. 3.3).  This library provides the steps of that path as
+ * device kernels behind plain C calls:
  *   logq_build_codebook  host: (bits, base, range) -> levels and boundaries
  *   logq_quantize        device: fp32 W[N][K] -> packed codes + codebook
  *   logq_quantize_energy device: the same with w_min / w_max / b derived from W
  *                        (Sec. 3.2, Eqs. (3)-(5))
+ *   logq_gptq_factor,    device: GPTQ calibration with the Log_b quantiser
+ *   logq_gptq            (the paper's post-training calibration): Hessian ->
+ *                        inverse-Hessian factor, then W -> packed codes
  *   logq_linear          device: codes, codebook, X[B][K] -> Y[B][N] = X * What^T
  *
  * Conventions shared by every call:
