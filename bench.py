@@ -639,7 +639,7 @@ def run_ours(args):
 
 
 CASES = ("gemv_gateup_1b", "gemv_gate_8b", "prefill_q_8b", "quantize_gate_8b", "energy_gate_8b",
-         "gemv8_gate_8b", "gptq_q_8b")
+         "gemv8_gate_8b", "gptq_q_8b", "gptq_update_q_8b")
 
 
 def run_case(name: str):
@@ -647,7 +647,8 @@ def run_case(name: str):
     the gate+up launch of the 1B decode step, the 8B gate GEMV, the 8B q-shaped
     prefill GEMM (2048 tokens), the quantisation of an 8B gate matrix, its
     self-calibrating (energy-range) quantisation, the 8-bit gate GEMV and 4-bit
-    GPTQ of an 8B q matrix (factor and quantisation)."""
+    GPTQ of an 8B q matrix (factor and quantisation; or the quantisation alone with a
+    fixed upper-triangular factor standing in for U)."""
     import torch
     import paper_2607_01127_gb300 as logq
     dev = torch.device("cuda", 0)
@@ -697,6 +698,19 @@ def run_case(name: str):
         cb = logq.logq_build_codebook(4, 1.5, float(W.abs().max()))
         for _ in range(2):
             logq.logq_gptq(W, H, cb)
+    elif name == "gptq_update_q_8b":
+        import ctypes
+        N, K = workloads.LLAMA_8B_SHAPES["q"]
+        W = workloads.weights_torch(N, K, 16, True, dev)
+        U = torch.triu(torch.full((K, K), 1e-3, device=dev)) + torch.eye(K, device=dev)
+        cb = logq.logq_build_codebook(4, 1.5, float(W.abs().max()))
+        codes = torch.empty(N * K // 2, dtype=torch.uint8, device=dev)
+        scratch = torch.empty(int(logq._lib().logq_gptq_scratch_bytes(N, K)), dtype=torch.uint8, device=dev)
+        for _ in range(2):
+            st = logq._lib().logq_gptq(ctypes.c_void_p(W.data_ptr()), N, K, ctypes.c_void_p(U.data_ptr()), None,
+                                       ctypes.byref(cb), ctypes.c_void_p(codes.data_ptr()),
+                                       ctypes.c_void_p(scratch.data_ptr()), scratch.numel(), None)
+            assert st == logq.LOGQ_OK
     torch.cuda.synchronize()
     st, _ = logq.logq_workspace_status(ws)
     assert st == logq.LOGQ_OK
