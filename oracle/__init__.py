@@ -15,7 +15,7 @@ Parity status of each function (what pins it is in ``tests/test_oracle.py``):
   quantize_*           pinned (three independent routes, level round trip,
                         idempotence, sign symmetry, base-2 frexp route)
   pack / unpack        pinned for the value set; the bit layout itself is a
-                        choice of this build ("parity unpinned" for the layout)
+                        choice of this library ("parity unpinned" for the layout)
   dequant              pinned through the codebook tables
   linear               pinned (float64 matmul of the dequantised weights,
                         one-hot and zero inputs)
