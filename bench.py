@@ -639,7 +639,7 @@ def run_ours(args):
 
 
 CASES = ("gemv_gateup_1b", "gemv_gate_8b", "prefill_q_8b", "quantize_gate_8b", "energy_gate_8b",
-         "gemv8_gate_8b", "gptq_q_8b", "gptq_update_q_8b")
+         "gemv8_gate_8b", "gptq_q_8b", "gptq_update_q_8b", "quantize3_gate_8b")
 
 
 def run_case(name: str):
@@ -677,6 +677,11 @@ def run_case(name: str):
         W = workloads.weights_torch(N, K, 15, True, dev)
         for _ in range(2):
             logq.logq_quantize(W, 4, 1.5, workspace=ws)
+    elif name == "quantize3_gate_8b":
+        N, K = workloads.LLAMA_8B_SHAPES["gate"]
+        W = workloads.weights_torch(N, K, 15, True, dev)
+        for _ in range(2):
+            logq.logq_quantize(W, 3, 1.8, workspace=ws)
     elif name == "gemv8_gate_8b":
         N, K = workloads.LLAMA_8B_SHAPES["gate"]
         c = logq.logq_quantize(workloads.weights_torch(N, K, 13, True, dev), 8, 1.04, workspace=ws)
