@@ -1,20 +1,23 @@
 """Benchmark of the Log_bQuant inference hot path on GB300.
 
-Workload (one step): the decode step of a Llama-3.2-1B-shaped model at batch
-1 -- all 16 layers x 7 linears (q/o 2048x2048, k/v 512x2048, gate/up
-8192x2048, down 2048x8192), 4-bit Log_b codes with a per-layer base drawn
-from U[1.2, 2.0], Student-t(4)*0.02 weights with 0.1 % x20 outliers, bf16
-activations, fp32 outputs.  Linears that read the same activations share a
-launch (q/k/v and gate/up through logq_linear_grouped), so a layer is four
-launches; each launch asks L2 to fetch the codes of the next one.  The 64
-launches of a step are captured once in a CUDA graph and replayed; the step's
-486 MB of codes exceed L2, so no flush is needed between steps.
+Workload (one step): the decode step of a Llama-3.1-8B-shaped model at batch
+1 -- all 32 layers x 7 linears (q/o 4096x4096, k/v 1024x4096, gate/up
+14336x4096, down 4096x14336), 4-bit Log_b codes with a per-layer base drawn
+from U[1.2, 2.0] and a per-tensor range max|W|, Student-t(4)*0.02 weights
+with 0.1 % x20 outliers, bf16 activations and outputs.  Linears that read the
+same activations share a launch (q/k/v and gate/up through
+logq_linear_grouped), so a layer is four launches; each launch asks L2 to
+fetch the codes of the next one.  The 128 launches of a step are captured once
+in a CUDA graph and replayed; the step's 3.49 GB of codes exceed L2, so no
+flush is needed between steps.  The Llama-3.2-1B-shaped step (16 layers, 64
+launches) is measured the same way as a second workload.
 
 metric: GEMV HBM GB/s at batch 1, counting the algorithmic bytes of every
 linear (packed codes + activations + outputs) per step.  The same run also
-measures the other rows of the path -- quantise (absmax + quantise + pack) of
-the whole model and the prefill GEMM on Llama-3.1-8B shapes (2048 tokens) --
-each with its own roofline, and times the fp64 oracle on the host cores.
+measures the other rows of the path -- the skinny GEMM at batch 4 and 16,
+quantise (absmax + quantise + pack), the prefill GEMM on Llama-3.1-8B shapes
+(2048 tokens) -- each with its own roofline, and times the fp64 oracle on the
+host cores.
 
 python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 N > 1 runs N independent replicas (one per GPU, launched by torchrun).
@@ -39,8 +42,15 @@ import numpy as np  # noqa: E402
 from paper_2607_01127_gb300 import workloads  # noqa: E402
 
 METRIC = "Log_b 4-bit GEMV HBM GB/s (% of ~8 TB/s) at batch 1; prefill GEMM TFLOP/s"
-WORKLOAD = "llama-3.2-1b decode step: 16 layers x {q,k,v,o,gate,up,down} 4-bit Log_b GEMV, batch 1"
-CFG_SEED = 1
+# decode-step workloads: layer shapes, layer count, seed of the configuration
+MODELS = {
+    "8b": dict(shapes=workloads.LLAMA_8B_SHAPES, layers=workloads.LLAMA_8B_LAYERS, cfg_seed=3,
+               name="llama-3.1-8b decode step: 32 layers x {q,k,v,o,gate,up,down} 4-bit Log_b GEMV, batch 1"),
+    "1b": dict(shapes=workloads.LLAMA_1B_SHAPES, layers=workloads.LLAMA_1B_LAYERS, cfg_seed=1,
+               name="llama-3.2-1b decode step: 16 layers x {q,k,v,o,gate,up,down} 4-bit Log_b GEMV, batch 1"),
+}
+HEADLINE = "8b"
+WORKLOAD = MODELS[HEADLINE]["name"]
 PREFILL_TOKENS = 2048
 
 
@@ -51,13 +61,14 @@ def peaks():
         return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
 
 
-def model_layers():
-    """(layer, proj, N, K, seed) for every linear of the 1B-shaped model."""
+def model_layers(model: str = HEADLINE):
+    """(layer, proj, N, K, seed) for every linear of the model."""
+    spec = MODELS[model]
     out = []
-    for layer in range(workloads.LLAMA_1B_LAYERS):
+    for layer in range(spec["layers"]):
         for pi, name in enumerate(workloads.PROJ_NAMES):
-            N, K = workloads.LLAMA_1B_SHAPES[name]
-            out.append((layer, name, N, K, workloads.layer_seed(CFG_SEED, layer, pi)))
+            N, K = spec["shapes"][name]
+            out.append((layer, name, N, K, workloads.layer_seed(spec["cfg_seed"], layer, pi)))
     return out
 
 
@@ -135,13 +146,14 @@ def traffic_for(kernel: str, source: str):
 
 # ----------------------------------------------------------------- oracle ---
 
-def oracle_gemv_sample(rows_per_layer: int = 8, seed: int = 0):
+def oracle_gemv_sample(rows_per_layer: int = 8, seed: int = 0, model: str = HEADLINE):
     """Inputs of the CPU baseline: the first rows of every linear of the model,
     quantised by the oracle (setup, untimed)."""
     import oracle
-    bases = workloads.layer_bases(workloads.LLAMA_1B_LAYERS, CFG_SEED)
+    spec = MODELS[model]
+    bases = workloads.layer_bases(spec["layers"], spec["cfg_seed"])
     items = []
-    for layer, name, N, K, s in model_layers():
+    for layer, name, N, K, s in model_layers(model):
         w = workloads.weights_np(rows_per_layer, K, s + seed, outliers=True)
         cb = oracle.build_codebook(4, float(bases[layer]), float(np.abs(w).max()))
         packed = oracle.pack(oracle.quantize_log(w, cb), 4)
@@ -171,8 +183,8 @@ def cpu_baseline(seconds: float = 12.0):
         reps += 1
     dt = time.perf_counter() - t0
     return {"value": round(nbytes / dt / 1e9, 4), "unit": "GB/s", "cores": threads, "kind": "oracle",
-            "sample": f"fp64 oracle GEMV over the first 8 rows of all 112 linears of the decode step, "
-                      f"{reps} passes in {dt:.1f} s"}
+            "sample": f"fp64 oracle GEMV over the first 8 rows of all {len(items)} linears of the decode "
+                      f"step, {reps} passes in {dt:.1f} s"}
 
 
 def run_reference(args):
@@ -196,7 +208,7 @@ def run_reference(args):
             "config": {"workload": WORKLOAD + " (oracle: first 8 rows of each linear per step)",
                        "l2": "n/a (host)"},
             "cpu_baseline": {"value": round(v, 4), "unit": "GB/s", "cores": threads, "kind": "oracle",
-                             "sample": "first 8 rows of each of the 112 linears per step"},
+                             "sample": f"first 8 rows of each of the {len(items)} linears per step"},
             "e2e": {"value": round(v, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -207,7 +219,7 @@ def run_reference(args):
 GROUPS = (("q", "k", "v"), ("o",), ("gate", "up"), ("down",))
 
 
-def build_decode_model(logq, torch, dev):
+def build_decode_model(logq, torch, dev, model: str = HEADLINE, layers: int | None = None):
     """Quantise every linear of the model into one contiguous code buffer (in
     launch order) and prepare the per-launch groups of the decode step.
 
@@ -216,24 +228,33 @@ def build_decode_model(logq, torch, dev):
     the launch before it (q -> o -> gate/up -> down -> the next layer's q/k/v;
     gate's output stands in for the activated MLP input of down).  So each
     launch depends on the previous one and finds its X in L2, as it would
-    after the attention / norm / activation kernels of a real model."""
-    bases = workloads.layer_bases(workloads.LLAMA_1B_LAYERS, CFG_SEED)
+    after the attention / norm / activation kernels of a real model.
+
+    Also counts the weights that lie within one fp32 ulp of a decision
+    boundary of their codebook (|w| equal to a boundary, rounded up to fp32,
+    or to the float just below it): the only weights whose code could depend
+    on how a boundary is rounded."""
+    spec = MODELS[model]
+    n_layers = spec["layers"] if layers is None else layers
+    bases = workloads.layer_bases(spec["layers"], spec["cfg_seed"])
     ws = logq.new_workspace(dev)
-    specs = model_layers()
+    specs = [x for x in model_layers(model) if x[0] < n_layers]
     total = sum(N * K // 2 for _, _, N, K, _ in specs)
     arena = torch.empty(total, dtype=torch.uint8, device=dev)
     lin = {}
     off = 0
+    near = 0
     for layer, name, N, K, s in specs:
         W = workloads.weights_torch(N, K, s, outliers=True, device=dev)
         nb = N * K // 2
         codes, cb = logq.logq_quantize(W, 4, float(bases[layer]), codes=arena[off:off + nb], workspace=ws)
+        near += boundary_neighbours(torch, W, cb)
         del W
         lin[(layer, name)] = dict(N=N, K=K, codes=codes, cb=cb, off=off, nbytes=nb, seed=s)
         off += nb
     launches = []
-    X = workloads.activations_torch(1, workloads.LLAMA_1B_SHAPES["q"][1], CFG_SEED, torch.bfloat16, dev)
-    for layer in range(workloads.LLAMA_1B_LAYERS):
+    X = workloads.activations_torch(1, spec["shapes"]["q"][1], spec["cfg_seed"], torch.bfloat16, dev)
+    for layer in range(n_layers):
         for grp in GROUPS:
             members = [lin[(layer, nm)] for nm in grp]
             K = members[0]["K"]
@@ -246,7 +267,16 @@ def build_decode_model(logq, torch, dev):
     for i, L in enumerate(launches):          # warm L2 with the next launch's codes
         nxt = launches[(i + 1) % len(launches)]
         L["pf"] = arena[nxt["off"]:nxt["off"] + nxt["nbytes"]]
-    return launches, ws, arena
+    stats = {"weights": sum(N * K for _, _, N, K, _ in specs), "boundary_neighbours": int(near)}
+    return launches, ws, arena, stats
+
+
+def boundary_neighbours(torch, W, cb) -> int:
+    """Weights of W whose magnitude is a decision boundary of cb (fp32, rounded up)
+    or the fp32 value just below one."""
+    t = torch.tensor([cb.thresh[j] for j in range(cb.qmax)], dtype=torch.float32, device=W.device)
+    cand = torch.cat([t, torch.nextafter(t, torch.zeros_like(t))])
+    return int(torch.isin(W.abs(), cand).sum().item())
 
 
 def linear_bytes_of(launch):
@@ -255,8 +285,8 @@ def linear_bytes_of(launch):
 
 
 def time_quantize(logq, torch, dev, reps: int = 2):
-    """Quantise every linear of the model (absmax pass + quantise-and-pack pass)."""
-    bases = workloads.layer_bases(workloads.LLAMA_1B_LAYERS, CFG_SEED)
+    """Quantise the first layer of the model (absmax pass + quantise-and-pack pass)."""
+    bases = workloads.layer_bases(MODELS[HEADLINE]["layers"], MODELS[HEADLINE]["cfg_seed"])
     ws = logq.new_workspace(dev)
     shapes = [(layer, N, K, s) for layer, name, N, K, s in model_layers()][:7]  # one layer, all shapes
     Ws = [workloads.weights_torch(N, K, s, outliers=True, device=dev) for _, N, K, s in shapes]
@@ -351,7 +381,7 @@ def time_gptq(logq, torch, dev):
     import ctypes
     N, K = workloads.LLAMA_8B_SHAPES["q"]
     W = workloads.weights_torch(N, K, workloads.layer_seed(4, 0, 0), outliers=True, device=dev)
-    g = torch.Generator(device=dev).manual_seed(CFG_SEED)
+    g = torch.Generator(device=dev).manual_seed(MODELS[HEADLINE]["cfg_seed"])
     X = torch.randn(3 * K, K, device=dev, generator=g, dtype=torch.float64)
     X[:, 1:] += 0.5 * X[:, :-1].clone()
     H64 = X.T @ X
@@ -445,6 +475,101 @@ def replica_totals(t_local: float, units_local: float, dist=None, device=None):
     return float(t.item()), float(u.item())
 
 
+def step_graph(logq, torch, launches, ws, stream, first_x=None):
+    """CUDA graph of one decode step (every launch of the chain, in order)."""
+    def run_launch(L, X=None):
+        items = [(m["codes"], m["cb"], m["N"], m["Y"]) for m in L["members"]]
+        logq.logq_linear_grouped(items, L["X"] if X is None else X, L["K"], y_dtype=torch.bfloat16,
+                                 workspace=ws, prefetch=L["pf"], prefetch_bytes=L["pf"].numel(), stream=stream)
+
+    def calls():
+        run_launch(launches[0], X=first_x)
+        for L in launches[1:]:
+            run_launch(L)
+
+    with torch.cuda.stream(stream):
+        calls()                                               # warm-up outside capture
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(stream):
+        with torch.cuda.graph(graph, stream=stream):
+            calls()
+    return graph
+
+
+def time_replays(torch, graph, stream, steps: int) -> float:
+    """Seconds for `steps` replays, CUDA events on the launching stream."""
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(steps):
+            graph.replay()
+        e1.record(stream)
+    e1.synchronize()
+    return e0.elapsed_time(e1) * 1e-3
+
+
+def time_decode_1b(logq, torch, dev, steps: int, warmup: int):
+    """The Llama-3.2-1B-shaped decode step, measured like the headline step."""
+    launches, ws, arena, _ = build_decode_model(logq, torch, dev, "1b")
+    stream = torch.cuda.Stream(device=dev)
+    graph = step_graph(logq, torch, launches, ws, stream)
+    for _ in range(warmup):
+        graph.replay()
+    torch.cuda.synchronize()
+    t = time_replays(torch, graph, stream, steps)
+    st, _ = logq.logq_workspace_status(ws)
+    assert st == logq.LOGQ_OK
+    step_bytes = sum(linear_bytes_of(L) for L in launches)
+    del graph, arena
+    return {"gbs": step_bytes * steps / t / 1e9, "ms_per_step": t / steps * 1e3, "launches": len(launches),
+            "bytes_per_step": step_bytes}
+
+
+def time_skinny(logq, torch, dev, batches=(1, 4, 16), reps: int = 10):
+    """Decode GEMV / skinny GEMM on the Llama-3.1-8B gate shape (14336 x 4096, 4-bit) at
+    several batch sizes, over rotating copies of the codes (more than L2 holds)."""
+    N, K = workloads.LLAMA_8B_SHAPES["gate"]
+    ws = logq.new_workspace(dev)
+    W = workloads.weights_torch(N, K, workloads.layer_seed(3, 0, 4), outliers=True, device=dev)
+    codes, cb = logq.logq_quantize(W, 4, 1.5, workspace=ws)
+    del W
+    copies = [codes] + [codes.clone() for _ in range(11)]          # 12 x 29.4 MB
+    s = torch.cuda.Stream(dev)
+    out = {}
+    for B in batches:
+        X = workloads.activations_torch(B, K, 3, torch.bfloat16, dev)
+        Y = torch.empty(B, N, dtype=torch.bfloat16, device=dev)
+
+        def launches():
+            for c in copies:
+                logq.logq_linear(c, cb, X, N, K, y_dtype=torch.bfloat16, Y=Y, workspace=ws, stream=s)
+        with torch.cuda.stream(s):
+            launches()
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(s):
+            with torch.cuda.graph(g, stream=s):
+                launches()
+        for _ in range(3):
+            g.replay()
+        torch.cuda.synchronize()
+        t = time_replays(torch, g, s, reps) / (reps * len(copies))
+        out[B] = {"us": t * 1e6, "gbs": linear_bytes(N, K, B=B, y_bytes=2) / t / 1e9,
+                  "tflops": 2.0 * B * N * K / t / 1e12}
+        del g
+    st, _ = logq.logq_workspace_status(ws)
+    assert st == logq.LOGQ_OK
+    return out
+
+
+def fp32_peak_tflops(sm_mhz: float) -> float:
+    """CUDA-core fp32 FMA rate: SMs x 128 lanes x 2 flops x clock."""
+    import torch
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    return sms * 128 * 2 * sm_mhz * 1e6 / 1e12
+
+
 def run_ours(args):
     import torch
     import paper_2607_01127_gb300 as logq
@@ -464,28 +589,12 @@ def run_ours(args):
             dist.barrier()
         torch.cuda.synchronize()
 
-    launches, ws, arena = build_decode_model(logq, torch, dev)
+    launches, ws, arena, stats = build_decode_model(logq, torch, dev)
     step_bytes = sum(linear_bytes_of(L) for L in launches)
     n_linears = sum(len(L["members"]) for L in launches)
     launches_per_step = len(launches)
     stream = torch.cuda.Stream(device=dev)
-
-    def run_launch(L, X=None):
-        items = [(m["codes"], m["cb"], m["N"], m["Y"]) for m in L["members"]]
-        logq.logq_linear_grouped(items, L["X"] if X is None else X, L["K"], y_dtype=torch.bfloat16,
-                                 workspace=ws, prefetch=L["pf"], prefetch_bytes=L["pf"].numel(), stream=stream)
-
-    def step_calls():
-        for L in launches:
-            run_launch(L)
-
-    with torch.cuda.stream(stream):
-        step_calls()                                          # warm-up outside capture
-    torch.cuda.synchronize()
-    graph = torch.cuda.CUDAGraph()
-    with torch.cuda.stream(stream):
-        with torch.cuda.graph(graph, stream=stream):
-            step_calls()
+    graph = step_graph(logq, torch, launches, ws, stream)
     for _ in range(args.warmup):
         graph.replay()
     barrier()
@@ -503,6 +612,8 @@ def run_ours(args):
     t, total_bytes = replica_totals(e0.elapsed_time(e1) * 1e-3, step_bytes * args.steps, dist, dev)
     value = total_bytes / t / 1e9
     ms_per_step = t / args.steps * 1e3
+    st, _ = logq.logq_workspace_status(ws, stream)
+    assert st == logq.LOGQ_OK, "decode step reported a device-side timeout"
 
     final = launches[-1]["members"][0]["Y"]
     y_device = final.clone()
@@ -515,19 +626,9 @@ def run_ours(args):
     yh = torch.empty(final.numel(), dtype=torch.bfloat16, pin_memory=True)
     xh.copy_(x0.view(-1).cpu())
     xd = torch.empty_like(x0)
-
-    def e2e_calls():
-        run_launch(launches[0], X=xd)
-        for L in launches[1:]:
-            run_launch(L)
-
-    g2 = torch.cuda.CUDAGraph()
     with torch.cuda.stream(stream):
         xd.copy_(xh.view(1, -1), non_blocking=True)
-        e2e_calls()
-        torch.cuda.synchronize()
-        with torch.cuda.graph(g2, stream=stream):
-            e2e_calls()
+    g2 = step_graph(logq, torch, launches, ws, stream, first_x=xd)
     h2d, d2h = xh.numel() * 2, yh.numel() * 2
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
@@ -548,11 +649,12 @@ def run_ours(args):
     # the step is deterministic: the end-to-end output equals the device-resident run
     assert torch.equal(yh.view(1, -1).to(dev), y_device)
     assert bool(torch.isfinite(y_device.float()).all())
+    del graph, g2, arena, launches
 
     pk, pk_kind = peaks()
     gemv_bytes_per_launch = step_bytes / launches_per_step
     achieved = gemv_bytes_per_launch / (t / args.steps / launches_per_step) / 1e9
-    tr = traffic_for("gemv_kernel", "paper_2607_01127_gb300/csrc/gemv.cu")
+    tr = traffic_for("gemv_kernel_8b_step", "paper_2607_01127_gb300/csrc/gemv.cu")
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": "GB/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4),
@@ -561,7 +663,7 @@ def run_ours(args):
         "config": {"workload": WORKLOAD, "global_batch": 1 * world, "linears_per_step": n_linears,
                    "launches_per_step": launches_per_step,
                    "bytes_per_step": step_bytes, "bits": 4,
-                   "l2": "inputs larger than L2 (486 MB of codes per step vs 126 MB L2)",
+                   "l2": f"inputs larger than L2 ({step_bytes / 1e9:.2f} GB of codes per step vs 126 MB L2)",
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                    "graph": "one CUDA graph per step: per layer qkv | o | gate+up | down launches "
                             "(linears that read the same activations share a launch), chained: each "
@@ -572,11 +674,38 @@ def run_ours(args):
         "gpu_launches": launches_per_step * args.steps,
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": pk["hbm_gbs"], "unit": "GB/s",
                      "frac": round(achieved / pk["hbm_gbs"], 4), "peak_source": pk_kind,
-                     "traffic": tr, "kernel": "gemv_kernel, batch 1, 4-bit (16 k per lane for q/k/v and o, 32 for gate/up and down)",
+                     "traffic": tr, "kernel": "gemv_kernel, batch 1, 4-bit (launches of the 8B step: 16-warp CTAs for gate+up and down, 8-warp CTAs for qkv and o)",
                      "algorithmic_bytes_per_launch": round(gemv_bytes_per_launch, 1),
                      "frac_of_8TBs": round(achieved / 8000.0, 4)},
+        "boundary_codes": {"within_1ulp_of_a_boundary": stats["boundary_neighbours"],
+                           "weights": stats["weights"],
+                           "note": "weights whose |w| is an fp32 decision boundary (rounded up) or the float "
+                                   "just below one: the only codes that depend on how a boundary is rounded"},
         "clocks": clocks.summary(),
     }
+    if rank == 0:
+        try:
+            d1 = time_decode_1b(logq, torch, dev, min(args.steps, 200), args.warmup)
+            line["decode_1b"] = {"gbs": round(d1["gbs"], 1), "frac": round(d1["gbs"] / pk["hbm_gbs"], 4),
+                                 "ms_per_step": round(d1["ms_per_step"], 4), "launches_per_step": d1["launches"],
+                                 "bytes_per_step": d1["bytes_per_step"],
+                                 "note": MODELS["1b"]["name"] + ", measured like the headline step"}
+        except Exception as e:
+            line["decode_1b"] = {"error": str(e)[:200]}
+        try:
+            sk = time_skinny(logq, torch, dev)
+            mhz = (line["clocks"] or {}).get("sm_mhz") or 2070.0
+            fp32 = fp32_peak_tflops(mhz)
+            line["skinny"] = {
+                f"B{B}": {"us": round(v["us"], 2), "gbs": round(v["gbs"], 1),
+                          "hbm_frac": round(v["gbs"] / pk["hbm_gbs"], 4), "tflops": round(v["tflops"], 2),
+                          "fp32_frac": round(v["tflops"] / fp32, 4)} for B, v in sk.items()}
+            line["skinny"]["fp32_peak_tflops"] = round(fp32, 1)
+            line["skinny"]["note"] = ("Llama-3.1-8B gate 14336x4096, 4-bit, bf16 in/out, 12 rotating code copies "
+                                      "(beyond L2); fp32_frac against SMs x 128 lanes x 2 flops x the median "
+                                      "SM clock of the headline run")
+        except Exception as e:
+            line["skinny"] = {"error": str(e)[:200]}
     if rank == 0:
         try:
             q = time_quantize(logq, torch, dev)
@@ -638,7 +767,7 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
-CASES = ("gemv_gateup_1b", "gemv_gate_8b", "prefill_q_8b", "quantize_gate_8b", "energy_gate_8b",
+CASES = ("decode_layers_8b", "gemv_gateup_1b", "gemv_gate_8b", "prefill_q_8b", "quantize_gate_8b", "energy_gate_8b",
          "gemv8_gate_8b", "gptq_q_8b", "gptq_update_q_8b", "quantize3_gate_8b")
 
 
@@ -653,7 +782,15 @@ def run_case(name: str):
     import paper_2607_01127_gb300 as logq
     dev = torch.device("cuda", 0)
     ws = logq.new_workspace(dev)
-    if name == "gemv_gateup_1b":
+    if name == "decode_layers_8b":
+        # the first two layers of the 8B decode step (8 chained launches, each
+        # warming L2 with the next one's codes), run twice
+        launches, ws, arena, _ = build_decode_model(logq, torch, dev, layers=2)
+        stream = torch.cuda.Stream(device=dev)
+        for _ in range(2):
+            step_graph(logq, torch, launches, ws, stream)
+        torch.cuda.synchronize()
+    elif name == "gemv_gateup_1b":
         K = 2048
         a = logq.logq_quantize(workloads.weights_torch(8192, K, 11, True, dev), 4, 1.4, workspace=ws)
         b = logq.logq_quantize(workloads.weights_torch(8192, K, 12, True, dev), 4, 1.6, workspace=ws)

@@ -304,7 +304,9 @@ typedef struct logq_linear_item {
  * l2_prefetch (device, may be NULL) / l2_prefetch_bytes name a range the
  * call asks the L2 cache to fetch while it runs -- for a decode step, the
  * codes of the next layer -- a hint only: it is never read by the
- * computation and may be any readable device memory.  Asynchronous; errors
+ * computation and may be any readable device memory at any alignment (the
+ * library prefetches the 16-byte aligned part inside it: the start rounded up
+ * and the length down to whole 16-byte units).  Asynchronous; errors
  * as logq_linear (LOGQ_ERR_INVALID_ARG also for count outside 1..4 or items
  * of different code widths).
  */

@@ -78,6 +78,19 @@ struct GroupArgs {
     Workspace* ws;
 };
 
+// The part of a prefetch hint [p, p + bytes) that a bulk L2 prefetch may take:
+// the start rounded up to 16 bytes and the length down to a multiple of 16 that
+// stays inside the range (*start = nullptr, *len = 0 when nothing is left).
+inline void aligned_prefetch_range(const void* p, size_t bytes, const void** start, int64_t* len)
+{
+    const uintptr_t p0 = reinterpret_cast<uintptr_t>(p);
+    const uintptr_t a = (p0 + 15u) & ~(uintptr_t)15u;
+    const size_t skip = (size_t)(a - p0);
+    const size_t n = (p && bytes > skip) ? ((bytes - skip) / 16) * 16 : 0;
+    *start = n > 0 ? reinterpret_cast<const void*>(a) : nullptr;
+    *len = (int64_t)n;
+}
+
 int sm_count();
 cudaError_t launch_absmax(const float* W, int64_t count, Workspace* ws, cudaStream_t s);
 cudaError_t launch_energy_range(const float* W, int64_t count, double eps, EnergyState* st, Workspace* ws,

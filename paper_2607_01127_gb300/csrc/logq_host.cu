@@ -369,8 +369,7 @@ logq_status logq_linear_grouped(const logq_linear_item* items, int count, const 
         g.bits = bits;
         g.x_f16 = x_f16;
         g.y_dtype = (int)y_dtype;
-        g.pf = l2_prefetch;
-        g.pf_bytes = (int64_t)((l2_prefetch_bytes / 16) * 16);
+        aligned_prefetch_range(l2_prefetch, l2_prefetch_bytes, &g.pf, &g.pf_bytes);
         g.ws = ws;
         return cuda_status(launch_gemv_group(g, s));
     }
