@@ -179,12 +179,14 @@ logq_status logq_linear(const uint8_t* codes, const logq_codebook* cb, const voi
  * that array until the process exits.  The scratch does not grow with N or K,
  * so the call accepts every size logq_quantize accepts (LOGQ_ERR_WORKSPACE would
  * report a scratch need beyond the array).  It calls no cudaMalloc, cudaFree
- * or other allocating routine.  Its first call on a device looks up the array's
- * device address (with that device current); make that first call before any
- * stream capture.  All calls share the one array, which keeps the last call's
- * contents (each call clears the words it needs): calls that overlap on the
- * GPU race and must be serialised by the caller.  Arguments, the single stream
- * synchronisation and the errors are otherwise those of logq_quantize.
+ * or other allocating routine.  Its first call on a device (and the first call
+ * after the device's context has been replaced, e.g. by cudaDeviceReset) looks
+ * up the array's device address with that device current; make that first call
+ * before any stream capture begins.  All calls share the one array, which
+ * keeps the last call's contents (each call clears the words it needs): calls
+ * that overlap on the GPU race and must be serialised by the caller.  Like
+ * logq_quantize it synchronises `stream` before returning; arguments and
+ * errors are those of logq_quantize, and the quantisation is the same code.
  */
 logq_status logq_quantize_noalloc(const float* W, int64_t N, int64_t K, int bits, double base,
                                   double range, int flags, uint8_t* codes,

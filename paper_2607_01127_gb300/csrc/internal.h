@@ -92,6 +92,13 @@ inline void aligned_prefetch_range(const void* p, size_t bytes, const void** sta
 }
 
 int sm_count();
+// logq_quantize after its workspace check: argument checks, and the
+// quantisation on a given workspace record (shared with the allocation-free
+// entry point, which passes its static record).
+logq_status check_quantize_args(const float* W, int64_t N, int64_t K, int bits, double base, double range,
+                                int flags, const uint8_t* codes);
+logq_status quantize_with(const float* W, int64_t N, int64_t K, int bits, double base, double range, int flags,
+                          uint8_t* codes, logq_codebook* cb_out, Workspace* ws, cudaStream_t s);
 cudaError_t launch_absmax(const float* W, int64_t count, Workspace* ws, cudaStream_t s);
 cudaError_t launch_energy_range(const float* W, int64_t count, double eps, EnergyState* st, Workspace* ws,
                                 cudaStream_t s);

@@ -26,6 +26,68 @@ int sm_count()
     return cached[dev];
 }
 
+// Argument checks shared by logq_quantize and logq_quantize_noalloc (all but
+// the scratch, which the two take from different places).
+logq_status check_quantize_args(const float* W, int64_t N, int64_t K, int bits, double base, double range,
+                                int flags, const uint8_t* codes)
+{
+    if (!W || !codes || (reinterpret_cast<uintptr_t>(W) & 15u) || (reinterpret_cast<uintptr_t>(codes) & 15u))
+        return LOGQ_ERR_INVALID_ARG;
+    if (logq_packed_bytes(N, K, bits) == 0) return LOGQ_ERR_INVALID_ARG;
+    if (!isfinite(base) || !(base > 1.0) || isnan(range) || isinf(range)) return LOGQ_ERR_INVALID_ARG;
+    if (flags != LOGQ_SHIFT_EXACT && flags != LOGQ_SHIFT_FLOOR) return LOGQ_ERR_INVALID_ARG;
+    if (N > (int64_t(1) << 40) / K) return LOGQ_ERR_INVALID_ARG;
+    return LOGQ_OK;
+}
+
+// The quantisation itself, on a workspace record ws (device): Sec. 3.2 w_max
+// when range <= 0, the codebook (Eqs. (2), (4)), then Eq. (1) and packing;
+// one 8-byte readback and one stream synchronisation report non-finite
+// weights.  Clears the two workspace words it uses first.
+logq_status quantize_with(const float* W, int64_t N, int64_t K, int bits, double base, double range, int flags,
+                          uint8_t* codes, logq_codebook* cb_out, Workspace* ws, cudaStream_t s)
+{
+    cudaError_t e = cudaMemsetAsync(ws, 0, 2 * sizeof(uint32_t), s);
+    if (e != cudaSuccess) return LOGQ_ERR_CUDA;
+
+    uint32_t host_words[2] = {0, 0};
+    const bool auto_range = !(range > 0.0);
+    if (auto_range) {
+        // Sec. 3.2: w_max = max_i |w_i|, reduced on the device.
+        if ((e = launch_absmax(W, N * K, ws, s)) != cudaSuccess) return LOGQ_ERR_CUDA;
+        if ((e = cudaMemcpyAsync(host_words, ws, sizeof host_words, cudaMemcpyDeviceToHost, s)) != cudaSuccess)
+            return LOGQ_ERR_CUDA;
+        if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return LOGQ_ERR_CUDA;
+        if (host_words[1]) return LOGQ_ERR_NONFINITE;
+        float mx;
+        memcpy(&mx, &host_words[0], 4);
+        if (!(mx > 0.0f)) return LOGQ_ERR_INVALID_ARG;   // all-zero weights: no log range
+        range = (double)mx;
+    }
+
+    logq_codebook cb;
+    logq_status st = logq_build_codebook(bits, base, range, flags, &cb);
+    if (st != LOGQ_OK) return st;
+
+    QuantParams p;
+    memset(&p, 0, sizeof p);
+    for (int j = 0; j < 128; ++j) p.thresh[j] = cb.thresh[j];
+    p.qmax = cb.qmax;
+    p.bits = bits;
+    p.check_nonfinite = auto_range ? 0 : 1;
+    if ((e = launch_quantize(W, N, K, p, codes, ws, s)) != cudaSuccess) return LOGQ_ERR_CUDA;
+    if (!auto_range) {
+        if ((e = cudaMemcpyAsync(host_words, ws, sizeof host_words, cudaMemcpyDeviceToHost, s)) != cudaSuccess)
+            return LOGQ_ERR_CUDA;
+        if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return LOGQ_ERR_CUDA;
+        if (host_words[1]) return LOGQ_ERR_NONFINITE;
+    } else {
+        if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return LOGQ_ERR_CUDA;
+    }
+    if (cb_out) *cb_out = cb;
+    return LOGQ_OK;
+}
+
 }  // namespace logq
 
 using namespace logq;
@@ -146,55 +208,12 @@ logq_status logq_quantize(const float* W, int64_t N, int64_t K, int bits, double
                           double range, int flags, uint8_t* codes, logq_codebook* cb_out,
                           void* workspace, size_t workspace_bytes, void* stream)
 {
-    if (!W || !codes || !aligned16(W) || !aligned16(codes)) return LOGQ_ERR_INVALID_ARG;
-    if (logq_packed_bytes(N, K, bits) == 0) return LOGQ_ERR_INVALID_ARG;
-    if (!isfinite(base) || !(base > 1.0) || isnan(range) || isinf(range)) return LOGQ_ERR_INVALID_ARG;
-    if (flags != LOGQ_SHIFT_EXACT && flags != LOGQ_SHIFT_FLOOR) return LOGQ_ERR_INVALID_ARG;
+    const logq_status st = check_quantize_args(W, N, K, bits, base, range, flags, codes);
+    if (st != LOGQ_OK) return st;
     if (!workspace || !aligned16(workspace) || workspace_bytes < kWorkspaceBytes)
         return LOGQ_ERR_WORKSPACE;
-    if (N > (int64_t(1) << 40) / K) return LOGQ_ERR_INVALID_ARG;
-
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
-    Workspace* ws = static_cast<Workspace*>(workspace);
-    cudaError_t e = cudaMemsetAsync(ws, 0, 2 * sizeof(uint32_t), s);
-    if (e != cudaSuccess) return LOGQ_ERR_CUDA;
-
-    uint32_t host_words[2] = {0, 0};
-    const bool auto_range = !(range > 0.0);
-    if (auto_range) {
-        // Sec. 3.2: w_max = max_i |w_i|, reduced on the device.
-        if ((e = launch_absmax(W, N * K, ws, s)) != cudaSuccess) return LOGQ_ERR_CUDA;
-        if ((e = cudaMemcpyAsync(host_words, ws, sizeof host_words, cudaMemcpyDeviceToHost, s)) != cudaSuccess)
-            return LOGQ_ERR_CUDA;
-        if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return LOGQ_ERR_CUDA;
-        if (host_words[1]) return LOGQ_ERR_NONFINITE;
-        float mx;
-        memcpy(&mx, &host_words[0], 4);
-        if (!(mx > 0.0f)) return LOGQ_ERR_INVALID_ARG;   // all-zero weights: no log range
-        range = (double)mx;
-    }
-
-    logq_codebook cb;
-    logq_status st = logq_build_codebook(bits, base, range, flags, &cb);
-    if (st != LOGQ_OK) return st;
-
-    QuantParams p;
-    memset(&p, 0, sizeof p);
-    for (int j = 0; j < 128; ++j) p.thresh[j] = cb.thresh[j];
-    p.qmax = cb.qmax;
-    p.bits = bits;
-    p.check_nonfinite = auto_range ? 0 : 1;
-    if ((e = launch_quantize(W, N, K, p, codes, ws, s)) != cudaSuccess) return LOGQ_ERR_CUDA;
-    if (!auto_range) {
-        if ((e = cudaMemcpyAsync(host_words, ws, sizeof host_words, cudaMemcpyDeviceToHost, s)) != cudaSuccess)
-            return LOGQ_ERR_CUDA;
-        if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return LOGQ_ERR_CUDA;
-        if (host_words[1]) return LOGQ_ERR_NONFINITE;
-    } else {
-        if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return LOGQ_ERR_CUDA;
-    }
-    if (cb_out) *cb_out = cb;
-    return LOGQ_OK;
+    return quantize_with(W, N, K, bits, base, range, flags, codes, cb_out, static_cast<Workspace*>(workspace),
+                         static_cast<cudaStream_t>(stream));
 }
 
 size_t logq_energy_scratch_bytes(void) { return sizeof(EnergyState); }

@@ -18,8 +18,13 @@ from gpu_common import lib
 
 pytestmark = pytest.mark.gpu
 
+# (N, K, bits, base, range, flags): 4-bit and 3-bit with the automatic range,
+# a given range with the floor shift, 8-bit codes (the 8-bit estimate kernel),
+# and bases outside the quantiser's estimate guards (1.05 at 4 bits, 1.005 at
+# 8 bits), which take the boundary-search kernels.
 CASES = [(512, 2048, 4, 1.5, 0.0, 0), (33, 1152, 3, 1.25, 0.0, 0), (64, 2048, 4, 2.0, 0.05, 1),
-         (300, 4096, 4, 1.7, 0.0, 0)]
+         (300, 4096, 4, 1.7, 0.0, 0), (96, 1024, 8, 1.04, 0.0, 0), (64, 512, 4, 1.05, 0.0, 0),
+         (40, 384, 8, 1.005, 0.0, 1)]
 
 
 def _cb_fields(cb):
