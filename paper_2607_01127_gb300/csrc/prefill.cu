@@ -75,6 +75,9 @@ constexpr long long kWaitLimit = 2000000000LL;   // cycles (~1 s)
 // error detail codes (workspace->detail)
 enum : uint32_t { kWaitProducer = 1, kWaitMma = 2, kWaitEpilogue = 3, kWaitDecode = 4, kWaitDrain = 5,
                   kWaitLayout = 6 };
+#ifdef LOGQ_TEST_WAIT_HOOK
+constexpr uint32_t kTestStallWord = 0x57A11u;   // workspace reserved[0] value that triggers the test stall
+#endif
 
 struct PrefillParams {
     const uint8_t* codes;
@@ -435,6 +438,14 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         uint32_t xph = 0, wph = 0;
         bool ok = true;
         int it = 0;
+#ifdef LOGQ_TEST_WAIT_HOOK
+        // Test builds only (never the shipped library): when the caller's
+        // workspace holds kTestStallWord, the MMA warp first waits on the drain
+        // barrier, which nothing completes before the teardown, so that wait
+        // runs out of its bound and the abort path of every role runs.
+        if (p.ws->reserved[0] == kTestStallWord)
+            ok = warp_wait(drainb, 0, abort_flag, p.ws, kWaitMma);
+#endif
         for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
             // one accumulator: the epilogue has read the previous tile's out of it
             if (!warp_wait(accempty, ((uint32_t)it & 1u) ^ 1u, abort_flag, p.ws, kWaitMma)) break;
