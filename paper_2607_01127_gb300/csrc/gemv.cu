@@ -22,7 +22,9 @@
 //    of the next launch on the stream: with programmatic dependent launch
 //    they start beside this one and build their table and issue their first
 //    code loads while it runs.  Large launches run one 16-warp CTA per SM to
-//    keep enough loads in flight; batches of 4 and more two 8-warp CTAs.
+//    keep enough loads in flight.  Batches of 4 and more hold more k per
+//    lane where registers allow (one CTA per SM), so that the cross-lane
+//    reduction of each row is shared by more multiply-adds.
 //  * The CTA's contiguous range of code rows is prefetched into L2 with bulk
 //    prefetches at kernel start, so HBM streams at full rate while the warps
 //    consume from L2.
@@ -311,8 +313,8 @@ __device__ __forceinline__ void decode_row(const CodeVec<NW>& c, uint32_t base_l
     }
 }
 
-template <int BITS, int B, int KW, int R, bool F16, int NT>
-__global__ void __launch_bounds__(NT, 512 / NT) gemv_kernel(const __grid_constant__ GemvParams p,
+template <int BITS, int B, int KW, int R, bool F16, int NT, int MINB = 512 / NT>
+__global__ void __launch_bounds__(NT, MINB) gemv_kernel(const __grid_constant__ GemvParams p,
                                                             const __grid_constant__ LevelsT<BITS> lv)
 {
     extern __shared__ __align__(16) uint8_t smem[];
@@ -567,7 +569,7 @@ struct Config {
 
 // Dynamic shared memory opt-in and a carveout that leaves room for two CTAs
 // per SM: per-device function attributes, set once per device.
-template <int BITS, int B, int KW, int R, bool F16, int NT>
+template <int BITS, int B, int KW, int R, bool F16, int NT, int MINB = 512 / NT>
 cudaError_t run(const GemvParams& p, const GroupArgs& a, int grid, size_t smem, cudaStream_t s)
 {
     LevelsT<BITS> lv;
@@ -575,7 +577,7 @@ cudaError_t run(const GemvParams& p, const GroupArgs& a, int grid, size_t smem, 
     if constexpr (BITS == 8)
         for (int i = 0; i < a.count; ++i)
             for (int c = 0; c < 256; ++c) lv.v[i][c] = a.item[i].lvl16[c];
-    auto k = gemv_kernel<BITS, B, KW, R, F16, NT>;
+    auto k = gemv_kernel<BITS, B, KW, R, F16, NT, MINB>;
     static bool configured[64] = {false};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -619,9 +621,14 @@ cudaError_t dispatch(int bits, int Bp, bool large, bool tiny, const GemvParams& 
             if (large) return run<4, 1, 32, 8, F16, L>(p, a, grid, smem, s);
             return tiny ? run<4, 1, 16, 8, F16, S>(p, a, grid, smem, s) : run<4, 1, 32, 8, F16, S>(p, a, grid, smem, s);
         case 2: return large ? run<4, 2, 32, 4, F16, L>(p, a, grid, smem, s) : run<4, 2, 32, 4, F16, S>(p, a, grid, smem, s);
-        case 4: return run<4, 4, 16, 2, F16, S>(p, a, grid, smem, s);
-        case 8: return run<4, 8, 8, 1, F16, S>(p, a, grid, smem, s);
-        case 16: return run<4, 16, 8, 1, F16, S>(p, a, grid, smem, s);
+        // batch 4: large launches one 16-warp CTA per SM with 32 k per lane,
+        // small ones two 8-warp CTAs with 16 k; batch 8 one 16-warp CTA with
+        // 16 k; batch 16 one 8-warp CTA whose threads hold 16 k of all 16
+        // activation rows (251 registers)
+        case 4: return large ? run<4, 4, 32, 2, F16, L, 1>(p, a, grid, smem, s)
+                             : run<4, 4, 16, 2, F16, S>(p, a, grid, smem, s);
+        case 8: return run<4, 8, 16, 1, F16, L, 1>(p, a, grid, smem, s);
+        case 16: return run<4, 16, 16, 1, F16, S, 1>(p, a, grid, smem, s);
         }
     } else {
         switch (Bp) {
@@ -642,12 +649,14 @@ int padded_batch(int64_t B)
     return 16;
 }
 
-int kw_for(int bits, int Bp, bool tiny)
+int kw_for(int bits, int Bp, bool tiny, bool large)
 {
     if (bits == 8) return 16;
     if (bits == 3) return 32;
     if (Bp == 1 && tiny) return 16;
-    return Bp <= 2 ? 32 : (Bp == 4 ? 16 : 8);
+    if (Bp <= 2) return 32;
+    if (Bp == 4) return large ? 32 : 16;
+    return 16;
 }
 
 // The table lookups address shared memory relative to kTabOff, which is where
@@ -687,7 +696,9 @@ cudaError_t launch_gemv_group(const GroupArgs& a, cudaStream_t s)
     for (int i = 0; i < a.count; ++i) total_rows += a.item[i].N;
     const int64_t row_bytes = (a.bits == 8) ? a.K : (a.bits == 4) ? a.K / 2 : a.K / 32 * 12;
     const bool tiny = a.bits == 4 && Bp == 1 && total_rows * row_bytes < kTinyBytes;
-    const int KW = kw_for(a.bits, Bp, tiny);
+    // large launches: batch 1-2 (and 4-bit batch 4) with at least kSplitBytes of codes
+    const bool large = (Bp <= 2 || (a.bits == 4 && Bp == 4)) && total_rows * row_bytes >= kSplitBytes;
+    const int KW = kw_for(a.bits, Bp, tiny, large);
     const int span = 32 * KW;
     GemvParams p;
     memset(&p, 0, sizeof p);
@@ -700,10 +711,11 @@ cudaError_t launch_gemv_group(const GroupArgs& a, cudaStream_t s)
     p.row_bytes = row_bytes;
     p.spans = (int32_t)((a.K + span - 1) / span);
     // Batch 1-2: large launches one 512-thread CTA per SM, small ones one
-    // 256-thread CTA per SM.  Batch 4 and more: two 256-thread CTAs per SM.
-    const bool large = Bp <= 2 && total_rows * p.row_bytes >= kSplitBytes;
-    const int threads = large ? kLargeThreads : kSmallThreads;
-    const int per_sm = Bp >= 4 ? 2 : 1;
+    // 256-thread CTA per SM.  3- and 8-bit batch 4: two 256-thread CTAs per SM;
+    // 4-bit batches of 4 and more: see dispatch() for the shapes.
+    const bool wide4 = a.bits == 4 && ((Bp == 4 && large) || Bp == 8);
+    const int threads = (large || wide4) ? kLargeThreads : kSmallThreads;
+    const int per_sm = (Bp >= 4 && !(a.bits == 4 && (Bp >= 8 || large))) ? 2 : 1;
     const int warps = threads / 32;
     if (p.spans >= warps) {
         p.groups = 1;

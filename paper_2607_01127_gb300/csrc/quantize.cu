@@ -240,49 +240,71 @@ __global__ void __launch_bounds__(256) quantize8e_kernel(const float4* __restric
     }
 }
 
-// 3-bit: each thread packs one group of 32 weights into 12 bytes.
+// 3-bit: each thread packs one group of 32 weights into three words (the
+// layout in logq.h).  A warp first copies its 32 consecutive groups (4 KiB) from
+// global memory with coalesced 16-byte loads (consecutive lanes on consecutive
+// 16 bytes) into its own shared-memory stage, and each lane then reads back its
+// group's eight 16-byte pieces; the stage is swizzled (piece q of group g at
+// g * 8 + (q ^ (g & 7))) so that both the stores and the reads are free of bank
+// conflicts.
 __global__ void __launch_bounds__(256) quantize3_kernel(const float4* __restrict__ W, int64_t ngroups,
                                                         QuantParams p, uint32_t* __restrict__ out,
                                                         Workspace* ws)
 {
+    __shared__ float4 stage[8][256];
     uint32_t t[8];
 #pragma unroll
     for (int j = 0; j < 8; ++j) t[j] = __float_as_uint(p.thresh[j]);
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    float4* st = stage[wid];
     uint32_t umax = 0;
-    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < ngroups; g += stride) {
-        uint32_t w0 = 0, w1 = 0, w2 = 0;
+    const int64_t wstride = (int64_t)gridDim.x * 8 * 32;          // groups per sweep of all warps
+    for (int64_t gb = ((int64_t)blockIdx.x * 8 + wid) * 32; gb < ngroups; gb += wstride) {
+        const int64_t left = ngroups - gb;
+        const int nf = (int)((left < 32 ? left : 32) * 8);         // 16-byte pieces of this batch
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {            // 4 weights = pairs 2q, 2q+1
-            const float4 a = ld_stream(W + 8 * g + q);
-            const float v[4] = {a.x, a.y, a.z, a.w};
-            uint32_t c[4];
+        for (int i = 0; i < 8; ++i) {
+            const int f = i * 32 + lane;
+            const int gl = f >> 3, q = f & 7;
+            st[gl * 8 + (q ^ (gl & 7))] = (f < nf) ? ld_stream(W + gb * 8 + f) : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+        __syncwarp();
+        if (lane < nf / 8) {
+            uint32_t w0 = 0, w1 = 0, w2 = 0;
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const uint32_t bits = __float_as_uint(v[e]);
-                const uint32_t u = bits & 0x7fffffffu;
-                umax = max(umax, u);
-                c[e] = code_of<3>(bits, magnitude<3>(u, t));
-            }
+            for (int q = 0; q < 8; ++q) {            // 4 weights = pairs 2q, 2q+1
+                const float4 a = st[lane * 8 + (q ^ (lane & 7))];
+                const float v[4] = {a.x, a.y, a.z, a.w};
+                uint32_t c[4];
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                const int pair = 2 * q + h;
-                const uint32_t f = c[2 * h] | (c[2 * h + 1] << 3);
-                if (pair < 15) {
-                    const uint32_t sh = f << (6 * (pair % 5));
-                    if (pair / 5 == 0) w0 |= sh;
-                    else if (pair / 5 == 1) w1 |= sh;
-                    else w2 |= sh;
-                } else {
-                    w0 |= (f & 3u) << 30;
-                    w1 |= ((f >> 2) & 3u) << 30;
-                    w2 |= ((f >> 4) & 3u) << 30;
+                for (int e = 0; e < 4; ++e) {
+                    const uint32_t bits = __float_as_uint(v[e]);
+                    const uint32_t u = bits & 0x7fffffffu;
+                    umax = max(umax, u);
+                    c[e] = code_of<3>(bits, magnitude<3>(u, t));
+                }
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int pair = 2 * q + h;
+                    const uint32_t f = c[2 * h] | (c[2 * h + 1] << 3);
+                    if (pair < 15) {
+                        const uint32_t sh = f << (6 * (pair % 5));
+                        if (pair / 5 == 0) w0 |= sh;
+                        else if (pair / 5 == 1) w1 |= sh;
+                        else w2 |= sh;
+                    } else {
+                        w0 |= (f & 3u) << 30;
+                        w1 |= ((f >> 2) & 3u) << 30;
+                        w2 |= ((f >> 4) & 3u) << 30;
+                    }
                 }
             }
+            const int64_t g = gb + lane;
+            out[3 * g + 0] = w0;
+            out[3 * g + 1] = w1;
+            out[3 * g + 2] = w2;
         }
-        out[3 * g + 0] = w0;
-        out[3 * g + 1] = w1;
-        out[3 * g + 2] = w2;
+        __syncwarp();                               // the stage is refilled next sweep
     }
     if (p.check_nonfinite) {
         const uint32_t bad = __reduce_or_sync(0xffffffffu, umax >= 0x7f800000u ? 1u : 0u);
@@ -442,7 +464,11 @@ cudaError_t launch_quantize(const float* W, int64_t N, int64_t K, const QuantPar
         }
     } else {
         const int64_t ngroups = total / 32;
-        quantize3_kernel<<<grid_for(ngroups, 256), 256, 0, s>>>(
+        // 32 KiB of staging per CTA: at most six resident per SM
+        const int sms = sm_count() > 0 ? sm_count() : 148;
+        int grid3 = grid_for(ngroups, 256);
+        if (grid3 > sms * 6) grid3 = sms * 6;
+        quantize3_kernel<<<grid3, 256, 0, s>>>(
             reinterpret_cast<const float4*>(W), ngroups, p, reinterpret_cast<uint32_t*>(codes), ws);
     }
     return cudaGetLastError();
