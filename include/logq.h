@@ -36,9 +36,14 @@
  *   - Decode launches (logq_linear with small B, logq_linear_grouped) use
  *     programmatic dependent launch: they may start while the preceding kernel
  *     on the stream finishes.  They read X and write Y only after that kernel
- *     has completed, but may read the packed codes earlier; codes written by
- *     a kernel that signals early completion (griddepcontrol.launch_dependents)
- *     must be ordered before the call by other means (e.g. an event or a copy).
+ *     has completed and its writes are visible, but they read the packed codes
+ *     earlier, before that guarantee holds.  So the codes must be complete
+ *     before the call is enqueued, ordered by a host synchronisation after the
+ *     kernel that wrote them (of its stream, of an event recorded after it, or
+ *     of the device), not by stream order alone.  logq_quantize and
+ *     logq_quantize_energy end with such a synchronisation; after logq_gptq
+ *     the caller synchronises.  Weights quantised once and reused (the decode
+ *     case) meet this.
  *   - Device code never traps.  Conditions found on the device (non-finite
  *     weights, a pipeline wait that exceeded its bound) are written to the
  *     caller's workspace and reported by logq_quantize or logq_workspace_status.
