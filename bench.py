@@ -767,7 +767,7 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
-CASES = ("decode_layers_8b", "gemv_gateup_1b", "gemv_gate_8b", "prefill_q_8b", "quantize_gate_8b", "energy_gate_8b",
+CASES = ("decode_layers_8b", "skinny_gate_8b", "gemv_gateup_1b", "gemv_gate_8b", "prefill_q_8b", "quantize_gate_8b", "energy_gate_8b",
          "gemv8_gate_8b", "gptq_q_8b", "gptq_update_q_8b", "quantize3_gate_8b")
 
 
@@ -790,6 +790,14 @@ def run_case(name: str):
         for _ in range(2):
             step_graph(logq, torch, launches, ws, stream)
         torch.cuda.synchronize()
+    elif name == "skinny_gate_8b":
+        # the 8B gate at batch 4 and 16, twice each
+        N, K = workloads.LLAMA_8B_SHAPES["gate"]
+        c = logq.logq_quantize(workloads.weights_torch(N, K, 13, True, dev), 4, 1.5, workspace=ws)
+        for B in (4, 16):
+            X = workloads.activations_torch(B, K, 1, torch.bfloat16, dev)
+            for _ in range(2):
+                logq.logq_linear(c[0], c[1], X, N, K, y_dtype=torch.bfloat16, workspace=ws)
     elif name == "gemv_gateup_1b":
         K = 2048
         a = logq.logq_quantize(workloads.weights_torch(8192, K, 11, True, dev), 4, 1.4, workspace=ws)

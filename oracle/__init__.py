@@ -27,6 +27,11 @@ Parity status of each function (what pins it is in ``tests/test_oracle.py``):
                         already quantised, solved directly; a dead input = the
                         reduced problem)
   base_from_range      pinned (closed form: q_max log steps span the range)
+  linear_asym          pinned (brute-force nearest of all 2^n grid values, uniform
+                        spacing, error bound, idempotence on its own grid, the
+                        scale^2 / 12 mean square error of uniform inputs); the
+                        comparison quantiser of the error study only, not part of the
+                        method
 """
 from __future__ import annotations
 
@@ -323,3 +328,23 @@ def bf16_bits_to_f64(bits: np.ndarray) -> np.ndarray:
 
 def f16_bits_to_f64(bits: np.ndarray) -> np.ndarray:
     return np.asarray(bits, dtype=np.uint16).view(np.float16).astype(np.float64)
+
+
+def linear_asym(w, bits: int, scale: float | None = None, zero: int | None = None):
+    """Tensor-wise asymmetric uniform (linear) quantisation with 2^bits levels: the
+    linear quantiser the paper contrasts Log_b with (Sec. 2 and Fig. 1: a uniform
+    grid spends its levels evenly over [min w, max w], while weight histograms are
+    bell-shaped), written from its standard definition in fp64:
+        scale = (max w - min w) / (2^bits - 1),   zero = round(-min w / scale),
+        q = clamp(round(w / scale) + zero, 0, 2^bits - 1),   value = (q - zero) * scale,
+    round() to nearest, ties to even.  scale and zero may be given (to requantise on a
+    fixed grid).  Returns (q, values, scale, zero).  Used only by the error study;
+    the library does not implement it."""
+    x = np.asarray(w, dtype=np.float64)
+    top = (1 << bits) - 1
+    if scale is None:
+        lo, hi = float(x.min()), float(x.max())
+        scale = (hi - lo) / top if hi > lo else 1.0
+        zero = int(np.rint(-lo / scale))
+    q = np.clip(np.rint(x / scale) + zero, 0, top).astype(np.int64)
+    return q, (q - zero).astype(np.float64) * scale, scale, zero

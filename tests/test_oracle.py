@@ -411,3 +411,45 @@ def test_gptq_factor_is_the_cholesky_factor_of_the_inverse(K):
         assert np.all(U[2, 3:] == 0.0) and np.all(U[:2, 2] == 0.0)
     assert np.all(np.tril(U, -1) == 0.0) and np.all(np.diag(U) > 0)
     np.testing.assert_allclose(U.T @ U @ Hd, np.eye(K), atol=1e-9)
+
+
+# ---------------------------------------------------------------- linear_asym ---
+# The comparison quantiser of the error study (tensor-wise asymmetric uniform).
+
+@pytest.mark.parametrize("bits", [3, 4, 8])
+def test_linear_asym_is_the_nearest_grid_value(bits):
+    """Brute force: each code is the nearest of all 2^n grid values (ties may go
+    either way), the grid is uniform with step scale, and no value errs by more than
+    half a step inside [min, max] except the top, which a rounded zero point can clip
+    by at most one step."""
+    rng = np.random.Generator(np.random.PCG64(bits))
+    w = rng.standard_t(4, size=2000) * 0.02
+    q, v, scale, zero = oracle.linear_asym(w, bits)
+    top = (1 << bits) - 1
+    grid = (np.arange(top + 1) - zero) * scale
+    d = np.abs(w[:, None] - grid[None, :])
+    best = d.min(axis=1)
+    assert np.allclose(np.abs(w - v), best, rtol=0, atol=1e-15)
+    assert np.allclose(np.diff(grid), scale)
+    assert np.isclose(scale, (w.max() - w.min()) / top)
+    inside = (w >= grid[0]) & (w <= grid[-1])
+    assert np.all(np.abs(w - v)[inside] <= scale / 2 + 1e-15)
+    assert np.all(np.abs(w - v) <= scale + 1e-15)
+
+
+@pytest.mark.parametrize("bits", [3, 4, 8])
+def test_linear_asym_idempotent_on_its_grid(bits):
+    w = workloads.weights_np(64, 64, 3 + bits, outliers=True).reshape(-1)
+    q, v, scale, zero = oracle.linear_asym(w, bits)
+    q2, v2, _, _ = oracle.linear_asym(v, bits, scale, zero)
+    assert np.array_equal(q, q2) and np.array_equal(v, v2)
+
+
+def test_linear_asym_uniform_mse_is_step_squared_over_12():
+    """For inputs spread uniformly over many grid steps the rounding error is uniform
+    on [-scale/2, scale/2]: mean square error scale^2 / 12."""
+    rng = np.random.Generator(np.random.PCG64(9))
+    w = rng.uniform(-1.0, 3.0, size=400_000)
+    _, v, scale, _ = oracle.linear_asym(w, 4)
+    mse = float(np.mean((w - v) ** 2))
+    assert abs(mse / (scale ** 2 / 12) - 1) < 0.02
