@@ -19,6 +19,7 @@
  *   logq_gptq            (the paper's post-training calibration): Hessian ->
  *                        inverse-Hessian factor, then W -> packed codes
  *   logq_linear          device: codes, codebook, X[B][K] -> Y[B][N] = X * What^T
+ *   logq_linear_grouped  the same for up to four matrices sharing X, one launch
  *
  * Conventions shared by every call:
  *   - Matrices are row-major and contiguous.  W and What are [N][K]
