@@ -674,7 +674,7 @@ def run_ours(args):
         "gpu_launches": launches_per_step * args.steps,
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": pk["hbm_gbs"], "unit": "GB/s",
                      "frac": round(achieved / pk["hbm_gbs"], 4), "peak_source": pk_kind,
-                     "traffic": tr, "kernel": "gemv_kernel, batch 1, 4-bit (launches of the 8B step: 16-warp CTAs for gate+up and down, 8-warp CTAs for qkv and o)",
+                     "traffic": tr, "kernel": "gemv_kernel, batch 1, 4-bit (the 128 launches of the 8B step: 8-warp CTAs, two per SM)",
                      "algorithmic_bytes_per_launch": round(gemv_bytes_per_launch, 1),
                      "frac_of_8TBs": round(achieved / 8000.0, 4)},
         "boundary_codes": {"within_1ulp_of_a_boundary": stats["boundary_neighbours"],

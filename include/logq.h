@@ -314,7 +314,9 @@ typedef struct logq_linear_item {
  * codes of the next layer -- a hint only: it is never read by the
  * computation and may be any readable device memory at any alignment (the
  * library prefetches the 16-byte aligned part inside it: the start rounded up
- * and the length down to whole 16-byte units).  Asynchronous; errors
+ * and the length down to whole 16-byte units).  A decode-GEMV launch ignores
+ * a range of 20 MiB or more: codes that large stream at full rate when their
+ * own launch reads them, and prefetching them would slow this one.  Asynchronous; errors
  * as logq_linear (LOGQ_ERR_INVALID_ARG also for count outside 1..4 or items
  * of different code widths).
  */

@@ -18,16 +18,17 @@
 //    reduce-scatter across the 32 lanes per round of rows, then a fixed-order
 //    sum over the spans in shared memory: results are bit-identical from run
 //    to run.
-//  * Small launches run one 8-warp CTA per SM, which leaves room for the CTAs
-//    of the next launch on the stream: with programmatic dependent launch
-//    they start beside this one and build their table and issue their first
-//    code loads while it runs.  Large launches run one 16-warp CTA per SM to
-//    keep enough loads in flight.  Batches of 4 and more hold more k per
-//    lane where registers allow (one CTA per SM), so that the cross-lane
-//    reduction of each row is shared by more multiply-adds.
-//  * The CTA's contiguous range of code rows is prefetched into L2 with bulk
-//    prefetches at kernel start, so HBM streams at full rate while the warps
-//    consume from L2.
+//  * Batch-1 4-bit launches run 8-warp CTAs, two per SM (tiny ones one per
+//    SM): with programmatic dependent launch, a CTA of the next launch on the
+//    stream starts as soon as one of them leaves, and builds its table and
+//    issues its first code loads while the rest of this launch finishes.
+//    Other small launches run one 8-warp CTA per SM (room for the next
+//    launch's CTAs), other large ones one 16-warp CTA per SM.  Batches of 4
+//    and more hold more k per lane where registers allow (one CTA per SM), so
+//    that the cross-lane reduction of each row is shared by more multiply-adds.
+//  * Where it pays, the CTA's contiguous range of code rows is prefetched into
+//    L2 with bulk prefetches at kernel start; an optional warm-up range (the
+//    next launch's codes) is prefetched the same way when it is small.
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <stdint.h>
@@ -40,9 +41,9 @@
 namespace logq {
 namespace {
 
-// Threads per CTA: 256 (two CTAs fit on an SM) for small launches and
-// batches of 4 and more, 512 (one per SM, all 16 warps sharing one table) for
-// large batch-1/2 launches.
+// Threads per CTA: 256 (two CTAs fit on an SM) for batch-1 4-bit launches,
+// small launches and batches of 4 and more, 512 (one per SM, all 16 warps
+// sharing one table) for the other large launches.
 constexpr int kSmallThreads = 256;
 constexpr int kLargeThreads = 512;
 constexpr int kTabStride = 256;               // bytes per pair-table entry
@@ -57,9 +58,11 @@ __host__ __device__ constexpr bool red_in_table(int bits, int B) { return bits =
 constexpr int64_t kPrefetchCap = 1 << 20;     // bytes of codes prefetched per CTA up front
 constexpr int kMaxSmem = 256 * kTabStride + kRedBytes;
 constexpr int kMaxItems = 4;
-// Launches with at least this many bytes of codes run 16 warps per SM: their
-// main loop needs them to keep enough loads in flight.  Smaller launches run
-// 8 warps per SM, leaving the other half of the SM to the next launch.
+// Launches with at least this many bytes of codes run 16 warps per SM (4-bit
+// batch 1: as two CTAs): their main loop needs them to keep enough loads in
+// flight.  Smaller launches run 8 warps per SM, leaving the other half of the
+// SM to the next launch.  Warm-up ranges of this size or more are not
+// prefetched.
 #ifndef LOGQ_GEMV_SPLIT_BYTES
 #define LOGQ_GEMV_SPLIT_BYTES (20 << 20)
 #endif
@@ -71,6 +74,16 @@ constexpr int64_t kSplitBytes = LOGQ_GEMV_SPLIT_BYTES;
 #define LOGQ_GEMV_TINY_BYTES (4 << 20)
 #endif
 constexpr int64_t kTinyBytes = LOGQ_GEMV_TINY_BYTES;
+// Tiny batch-1 4-bit launches: CTAs per SM, and whether they prefetch their
+// own code rows into L2 (one CTA per SM with the prefetch measured best on the
+// 1B decode step; every other batch-1 4-bit launch runs two per SM without it).
+#ifndef LOGQ_GEMV_TINY_PER_SM
+#define LOGQ_GEMV_TINY_PER_SM 1
+#endif
+constexpr int kTinyPerSm = LOGQ_GEMV_TINY_PER_SM;
+#ifndef LOGQ_GEMV_TINY_OWN_PF
+#define LOGQ_GEMV_TINY_OWN_PF 1
+#endif
 // Shared-memory carveout of the batch-1/2 decode kernels, in percent of the
 // maximum: 58 % is 132 KiB, room for two CTAs of 64 KiB (plus their reserved
 // 1 KiB).  The rest of the 256 KiB per SM is L1, which also holds the data of
@@ -110,6 +123,8 @@ struct GemvParams {
     const uint8_t* pf;    // optional L2 warm-up range (e.g. the next layer's codes)
     int64_t pf_bytes;
     int64_t pf_share;     // bytes of that range per CTA (multiple of 16)
+    int32_t own_pf;       // prefetch the CTA's own code rows into L2 at start
+    int32_t _pad;
 };
 
 // 8-bit codes: their 256 code-indexed levels per matrix travel as a second
@@ -390,7 +405,7 @@ __global__ void __launch_bounds__(NT, MINB) gemv_kernel(const __grid_constant__ 
     {
         constexpr int64_t piece = 16384;
         const uint8_t* base = item.codes + r0 * p.row_bytes;
-        int64_t bytes = (r1 - r0) * p.row_bytes;
+        int64_t bytes = p.own_pf ? (r1 - r0) * p.row_bytes : 0;
         if (bytes > kPrefetchCap) bytes = kPrefetchCap;
         for (int64_t off = (int64_t)tid * piece; off < bytes; off += (int64_t)NT * piece) {
             const int64_t n = (bytes - off) < piece ? (bytes - off) : piece;
@@ -617,9 +632,10 @@ cudaError_t dispatch(int bits, int Bp, bool large, bool tiny, const GemvParams& 
         }
     } else if (bits == 4) {
         switch (Bp) {
+        // batch 1: 8-warp CTAs, two per SM (tiny launches: one per SM)
         case 1:
-            if (large) return run<4, 1, 32, 8, F16, L>(p, a, grid, smem, s);
-            return tiny ? run<4, 1, 16, 8, F16, S>(p, a, grid, smem, s) : run<4, 1, 32, 8, F16, S>(p, a, grid, smem, s);
+            return tiny ? run<4, 1, 16, 8, F16, S, kTinyPerSm>(p, a, grid, smem, s)
+                        : run<4, 1, 32, 8, F16, S, 2>(p, a, grid, smem, s);
         case 2: return large ? run<4, 2, 32, 4, F16, L>(p, a, grid, smem, s) : run<4, 2, 32, 4, F16, S>(p, a, grid, smem, s);
         // batch 4: large launches one 16-warp CTA per SM with 32 k per lane,
         // small ones two 8-warp CTAs with 16 k; batch 8 one 16-warp CTA with
@@ -714,8 +730,10 @@ cudaError_t launch_gemv_group(const GroupArgs& a, cudaStream_t s)
     // 256-thread CTA per SM.  3- and 8-bit batch 4: two 256-thread CTAs per SM;
     // 4-bit batches of 4 and more: see dispatch() for the shapes.
     const bool wide4 = a.bits == 4 && ((Bp == 4 && large) || Bp == 8);
-    const int threads = (large || wide4) ? kLargeThreads : kSmallThreads;
-    const int per_sm = (Bp >= 4 && !(a.bits == 4 && (Bp >= 8 || large))) ? 2 : 1;
+    const bool b1_4 = a.bits == 4 && Bp == 1;
+    const int threads = ((large && !b1_4) || wide4) ? kLargeThreads : kSmallThreads;
+    const int per_sm = b1_4 ? (tiny ? kTinyPerSm : 2)
+                            : (Bp >= 4 && !(a.bits == 4 && (Bp >= 8 || large))) ? 2 : 1;
     const int warps = threads / 32;
     if (p.spans >= warps) {
         p.groups = 1;
@@ -724,8 +742,15 @@ cudaError_t launch_gemv_group(const GroupArgs& a, cudaStream_t s)
         p.groups = warps / p.spans;
         p.span_cols = p.spans;
     }
+    // Each CTA's own rows are prefetched into L2 up front only where that was
+    // measured to pay: not in 4-bit batch-1 launches (two CTAs per SM, whose
+    // code loads keep enough in flight) except tiny ones, nor in large launches.
+    p.own_pf = b1_4 ? (tiny ? LOGQ_GEMV_TINY_OWN_PF : 0) : (large ? 0 : 1);
+    // The warm-up range is prefetched only when it is below kSplitBytes: a
+    // launch that large streams its own codes at full rate, and warming L2
+    // with them slows the launch that issues the prefetch more than it helps.
     p.pf = static_cast<const uint8_t*>(a.pf);
-    p.pf_bytes = a.pf ? a.pf_bytes : 0;
+    p.pf_bytes = (a.pf && a.pf_bytes < kSplitBytes) ? a.pf_bytes : 0;
 
     // CTAs in proportion to each matrix's rows (at least one each, at most one
     // per row).
