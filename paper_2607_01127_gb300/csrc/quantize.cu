@@ -312,6 +312,107 @@ __global__ void __launch_bounds__(256) quantize3_kernel(const float4* __restrict
     }
 }
 
+// 3-bit with the level estimated as in quantize4e_kernel (q_max = 3; the same
+// fixed point and guards).  Each warp streams batches of 32 consecutive groups
+// (4 KiB) into two alternating shared-memory stages with asynchronous 16-byte
+// copies (swizzled as in quantize3_kernel), so the next batch is in flight while
+// the lanes code the current one.  Each weight adds m + 4 * sign into its 3-bit
+// slot of the group's word (weights 0-29: word e / 10, slot e % 10, which is the
+// layout's field of pair e / 2); the sign is then cleared in every slot whose
+// magnitude is 0 at once: (m + 3) carries into the slot's bit 2 exactly when
+// m != 0, and never out of the slot.  Weights 30 and 31 (pair 15, split over
+// the three words' top bits) are coded one by one.  The codes equal
+// quantize3_kernel's bit for bit.
+constexpr int kQ3eThreads = 128;
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+
+template <bool CHECK>
+__global__ void __launch_bounds__(kQ3eThreads) quantize3e_kernel(const float4* __restrict__ W, int64_t ngroups,
+                                                                 const __grid_constant__ QuantEst q,
+                                                                 uint32_t* __restrict__ out, Workspace* ws)
+{
+    constexpr int kWarps = kQ3eThreads / 32;
+    __shared__ float4 stage[kWarps][2][256];
+    __shared__ uint32_t t2[4];
+    if (threadIdx.x < 4) t2[threadIdx.x] = q.t2[threadIdx.x];
+    __syncthreads();
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    uint32_t umax = 0;                                             // largest 2|w| bit pattern seen
+    constexpr uint32_t kLow = 0x1B6DB6DBu;                        // 0b011 in each of 10 slots
+    constexpr uint32_t kBit2 = 0x24924924u;                       // 0b100 in each of 10 slots
+    const int64_t wstride = (int64_t)gridDim.x * kWarps * 32;     // groups per sweep of all warps
+    // copies of the batch at gb into stage b (pieces past the end are not copied:
+    // only lanes whose group exists read the stage)
+    auto issue = [&](int b, int64_t gb) {
+        const int64_t left = ngroups - gb;
+        const int nf = (int)((left < 32 ? left : 32) * 8);
+        const uint32_t base = (uint32_t)__cvta_generic_to_shared(&stage[wid][b][0]);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            const int f = i * 32 + lane;
+            const int gl = f >> 3, qq = f & 7;
+            if (f < nf) cp_async16(base + 16u * (uint32_t)(gl * 8 + (qq ^ (gl & 7))), W + gb * 8 + f);
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    };
+    int64_t gb = ((int64_t)blockIdx.x * kWarps + wid) * 32;
+    if (gb < ngroups) issue(0, gb);
+    for (int b = 0; gb < ngroups; b ^= 1) {
+        const int64_t gn = gb + wstride;
+        if (gn < ngroups) issue(b ^ 1, gn);
+        else asm volatile("cp.async.commit_group;" ::: "memory");   // keeps one group per batch
+        asm volatile("cp.async.wait_group 1;" ::: "memory");         // this batch has landed
+        __syncwarp();
+        const float4* st = stage[wid][b];
+        const int64_t left = ngroups - gb;
+        if (lane < (left < 32 ? left : 32)) {
+            uint32_t v[3] = {0u, 0u, 0u};
+            uint32_t c30 = 0, c31 = 0;
+#pragma unroll
+            for (int qq = 0; qq < 8; ++qq) {
+                const float4 a = st[lane * 8 + (qq ^ (lane & 7))];
+                const float w4[4] = {a.x, a.y, a.z, a.w};
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int e = 4 * qq + i;
+                    const uint32_t bits = __float_as_uint(w4[i]);
+                    const uint32_t u2 = bits << 1;                  // 2|w|: the sign bit drops out
+                    if (CHECK) umax = max(umax, u2);
+                    const uint64_t pe = (uint64_t)u2 * q.K + q.C;
+                    const int mh = __vimin_s32_relu((int)(uint32_t)(pe >> 32), 3);
+                    const uint32_t val = (uint32_t)mh + (u2 >= t2[mh] ? 1u : 0u) + ((bits >> 31) << 2);
+                    if (e < 30) v[e / 10] += val << (3 * (e % 10));  // disjoint slots: add = or
+                    else if (e == 30) c30 = val;
+                    else c31 = val;
+                }
+            }
+#pragma unroll
+            for (int j = 0; j < 3; ++j) {
+                const uint32_t lo = v[j] & kLow;
+                v[j] = lo | (v[j] & ((lo + kLow) & kBit2));
+            }
+            c30 = (c30 & 3u) | (c30 & (((c30 & 3u) + 3u) & 4u));
+            c31 = (c31 & 3u) | (c31 & (((c31 & 3u) + 3u) & 4u));
+            const uint32_t f15 = c30 | (c31 << 3);
+            const int64_t g = gb + lane;
+            out[3 * g + 0] = v[0] | ((f15 & 3u) << 30);
+            out[3 * g + 1] = v[1] | (((f15 >> 2) & 3u) << 30);
+            out[3 * g + 2] = v[2] | (((f15 >> 4) & 3u) << 30);
+        }
+        __syncwarp();                                  // stage b is refilled two batches on
+        gb = gn;
+    }
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+    if (CHECK) {
+        const uint32_t bad = __reduce_or_sync(0xffffffffu, umax >= 0xff000000u ? 1u : 0u);
+        if (bad && (threadIdx.x & 31) == 0) atomicOr(&ws->nonfinite, 1u);
+    }
+}
+
 // 8-bit: each thread turns 16 consecutive weights into 16 code bytes.  The
 // 127 boundaries live in shared memory (as bit patterns, with +Inf appended)
 // and a seven-step binary search counts those not above |w|.
@@ -354,8 +455,9 @@ __global__ void __launch_bounds__(256) quantize8_kernel(const float4* __restrict
     }
 }
 
-// Fixed-point slope and offset of quantize4e_kernel's level estimate, from the
-// 4-bit boundaries; false when the guards fail (the boundary search is used).
+// Fixed-point slope and offset of the level estimate of quantize4e_kernel and
+// quantize3e_kernel, from the 4-bit (q_max = 7) or 3-bit (q_max = 3)
+// boundaries; false when the guards fail (the boundary search is used).
 //   lambda = log2 of the boundary ratio, from the first and last boundary;
 //   estimate(u2) = floor((u2 K + C) / 2^32) with K = round(2^8 / lambda) and
 //   C = round(-(log2 t_0 + 127) 2^24 K + (1 - 0.05) 2^32), i.e. the level count
@@ -365,21 +467,22 @@ __global__ void __launch_bounds__(256) quantize8_kernel(const float4* __restrict
 //   0.0861 / lambda <= 0.72 levels for lambda >= 0.12.
 bool estimate_params(const QuantParams& p, QuantEst& q)
 {
-    if (p.bits != 4 || p.qmax != 7) return false;
-    const double t0 = p.thresh[0], t6 = p.thresh[6];
-    if (!(t0 >= 1.1754943508222875e-38) || !(t6 > t0) || !isfinite(t6)) return false;
+    if (!((p.bits == 4 && p.qmax == 7) || (p.bits == 3 && p.qmax == 3))) return false;
+    const int last = p.qmax - 1;
+    const double t0 = p.thresh[0], tl = p.thresh[last];
+    if (!(t0 >= 1.1754943508222875e-38) || !(tl > t0) || !isfinite(tl)) return false;
     const double l0 = log2(t0);
-    const double lambda = (log2(t6) - l0) / 6.0;
+    const double lambda = (log2(tl) - l0) / (double)last;
     if (!(lambda >= 0.12) || !(lambda <= 3.0)) return false;
     const double k = nearbyint(256.0 / lambda);
     q.K = (uint32_t)k;
     q.C = (uint64_t)(int64_t)nearbyint(-(l0 + 127.0) * 16777216.0 * k + 0.95 * 4294967296.0);
-    for (int j = 0; j < 7; ++j) {
-        uint32_t b;
-        memcpy(&b, &p.thresh[j], 4);
-        q.t2[j] = 2u * b;
+    for (int j = 0; j < 8; ++j) {
+        uint32_t b = 0;
+        if (j < p.qmax) memcpy(&b, &p.thresh[j], 4);
+        q.t2[j] = j < p.qmax ? 2u * b : 0xffffffffu;
     }
-    q.t2[7] = 0xffffffffu;
+    q._pad = 0;
     return true;
 }
 
@@ -468,8 +571,21 @@ cudaError_t launch_quantize(const float* W, int64_t N, int64_t K, const QuantPar
         const int sms = sm_count() > 0 ? sm_count() : 148;
         int grid3 = grid_for(ngroups, 256);
         if (grid3 > sms * 6) grid3 = sms * 6;
-        quantize3_kernel<<<grid3, 256, 0, s>>>(
-            reinterpret_cast<const float4*>(W), ngroups, p, reinterpret_cast<uint32_t*>(codes), ws);
+        QuantEst q;
+        if (estimate_params(p, q)) {
+            // 32 KiB of stages per 128-thread CTA: six resident per SM
+            int grid3e = (int)((ngroups + kQ3eThreads - 1) / kQ3eThreads);
+            if (grid3e > sms * 6) grid3e = sms * 6;
+            if (p.check_nonfinite)
+                quantize3e_kernel<true><<<grid3e, kQ3eThreads, 0, s>>>(
+                    reinterpret_cast<const float4*>(W), ngroups, q, reinterpret_cast<uint32_t*>(codes), ws);
+            else
+                quantize3e_kernel<false><<<grid3e, kQ3eThreads, 0, s>>>(
+                    reinterpret_cast<const float4*>(W), ngroups, q, reinterpret_cast<uint32_t*>(codes), ws);
+        } else {
+            quantize3_kernel<<<grid3, 256, 0, s>>>(
+                reinterpret_cast<const float4*>(W), ngroups, p, reinterpret_cast<uint32_t*>(codes), ws);
+        }
     }
     return cudaGetLastError();
 }

@@ -75,11 +75,12 @@ def test_quantize_special_values(logq):
 
 @pytest.mark.parametrize("bad", [np.nan, np.inf, -np.inf])
 @pytest.mark.parametrize("given_range", [0.0, 1.0])
-def test_quantize_nonfinite_reported(logq, bad, given_range):
+@pytest.mark.parametrize("bits", [3, 4])
+def test_quantize_nonfinite_reported(logq, bad, given_range, bits):
     w = workloads.weights_np(16, 256, 5)
     w[3, 17] = bad
     with pytest.raises(logq.LogqError) as ei:
-        logq.logq_quantize(torch.from_numpy(w).cuda(), 4, 1.5, given_range)
+        logq.logq_quantize(torch.from_numpy(w).cuda(), bits, 1.5, given_range)
     assert ei.value.status == logq.LOGQ_ERR_NONFINITE
     # the context stays usable
     codes, _ = logq.logq_quantize(torch.from_numpy(np.nan_to_num(w, posinf=0, neginf=0)).cuda(), 4, 1.5)
@@ -104,13 +105,14 @@ def test_quantize_repeatable(logq):
 
 @pytest.mark.parametrize("base", [1.05, 1.087, 1.1, 1.5, 3.0, 7.9, 9.0])
 @pytest.mark.parametrize("mode", [0, 1])
-def test_quantize4_every_boundary_and_neighbours(logq, base, mode):
-    """4-bit codes of every fp32 boundary, its two fp32 neighbours on each side, both
-    signs, subnormals, zeros and values far outside the range: bit-exact.  Bases from
-    1.05 to 9 cover the boundary search and the estimate-and-correct kernel (used for
-    boundary ratios 2^0.12 to 2^3) on both sides of its guards."""
+@pytest.mark.parametrize("bits", [3, 4])
+def test_quantize_every_boundary_and_neighbours(logq, base, mode, bits):
+    """3- and 4-bit codes of every fp32 boundary, its two fp32 neighbours on each side,
+    both signs, subnormals, zeros and values far outside the range: bit-exact.  Bases
+    from 1.05 to 9 cover the boundary search and the estimate-and-correct kernels (used
+    for boundary ratios 2^0.12 to 2^3) on both sides of their guards."""
     rng_ = 0.75
-    ocb = oracle.build_codebook(4, base, rng_, mode)
+    ocb = oracle.build_codebook(bits, base, rng_, mode)
     t = np.asarray(ocb.taus32_up, np.float32)
     near = np.concatenate([t, np.nextafter(t, np.float32(0)), np.nextafter(t, np.float32(np.inf)),
                            np.nextafter(np.nextafter(t, np.float32(0)), np.float32(0)),
@@ -120,5 +122,5 @@ def test_quantize4_every_boundary_and_neighbours(logq, base, mode):
     rnd = (np.random.default_rng(int(base * 1000) + mode).standard_normal(128 * 64) * 0.3).astype(np.float32)
     w = np.concatenate([near, -near, extra, rnd]).astype(np.float32)
     w = np.concatenate([w, np.zeros((-w.size) % 128, np.float32)]).reshape(-1, 128)
-    codes, cb = logq.logq_quantize(torch.from_numpy(w).cuda(), 4, base, rng_, mode)
-    assert check_codes(codes.cpu().numpy(), w, ocb, 4) == 0
+    codes, cb = logq.logq_quantize(torch.from_numpy(w).cuda(), bits, base, rng_, mode)
+    assert check_codes(codes.cpu().numpy(), w, ocb, bits) == 0
