@@ -545,21 +545,46 @@ __global__ void __launch_bounds__(NT, MINB) gemv_kernel(const __grid_constant__ 
                         run1(cb, t + 1);
                     }
                 } else {
+                    // Full rounds run without any row checks (branches and their
+                    // convergence points were a quarter of the loop's
+                    // instructions); only the last, partial round checks its rows.
+                    // ca holds round 0 (full, or the partial round itself).
+                    const int nfull = my_rows / R, tail = my_rows - nfull * R;
+                    const int64_t rstep = (int64_t)R * rstride;
+                    auto load_full = [&](CodeVec<NW> (&c)[R], const uint8_t* rp) {
+#pragma unroll
+                        for (int r = 0; r < R; ++r) c[r] = ld_codes<NW>(rp + r * rstride);
+                    };
+                    auto run_full = [&](const CodeVec<NW> (&c)[R]) {
+                        float acc[V], acc_hi[V];
+#pragma unroll
+                        for (int i = 0; i < V; ++i) acc[i] = acc_hi[i] = 0.f;
+#pragma unroll
+                        for (int r = 0; r < R; ++r)
+                            decode_row<BITS, B, NW, F16>(c[r], base_lane, xr, acc + r * B, acc_hi + r * B);
+#pragma unroll
+                        for (int i = 0; i < V; ++i) acc[i] += acc_hi[i];
+                        reduce_scatter<V>(acc, lane);
+                        if (writer) red(red_i) = acc[0];            // a full round's rows all exist
+                        lr_w += G * R;
+                        red_i += G * R * B;
+                    };
                     const uint8_t* rp = first;
-                    int here = my_rows;               // rows of this warp from round rp on
-                    while (true) {
-                        const uint8_t* rn = rp + R * rstride;
-                        if (here > R) load_round(cb, rn, here - R);
-                        run_round(ca, here);
-                        if (here <= R) break;
-                        rp = rn;
-                        here -= R;
-                        rn = rp + R * rstride;
-                        if (here > R) load_round(ca, rn, here - R);
-                        run_round(cb, here);
-                        if (here <= R) break;
-                        rp = rn;
-                        here -= R;
+                    int t = 0;
+                    for (; t + 2 <= nfull; t += 2) {                // rounds t (in ca) and t + 1
+                        load_full(cb, rp + rstep);
+                        run_full(ca);
+                        if (t + 2 < nfull) load_full(ca, rp + 2 * rstep);
+                        else if (tail) load_round(ca, rp + 2 * rstep, tail);
+                        run_full(cb);
+                        rp += 2 * rstep;
+                    }
+                    if (t < nfull) {                                 // one full round left, in ca
+                        if (tail) load_round(cb, rp + rstep, tail);
+                        run_full(ca);
+                        if (tail) run_round(cb, tail);
+                    } else if (tail) {
+                        run_round(ca, tail);
                     }
                 }
             }
