@@ -139,6 +139,16 @@ size_t logq_packed_bytes(int64_t N, int64_t K, int bits);
  * same time on different streams need separate workspaces. */
 size_t logq_workspace_bytes(void);
 
+/* Bytes of workspace with which logq_linear (and logq_linear_grouped, per
+ * matrix) runs a B x N x K product at full speed: logq_workspace_bytes() plus,
+ * for products that run on the tensor cores, room for fp32 partial sums when
+ * the output tiles are too few to fill the GPU and each tile's k range is split
+ * over several CTAs (Y is then their fixed-order sum, a second kernel on the
+ * same stream).  A smaller workspace (at least logq_workspace_bytes()) is
+ * accepted: the call then splits less, or, for 4-bit batches of 8..16, keeps
+ * the CUDA-core kernel.  0 for invalid sizes. */
+size_t logq_linear_workspace_bytes(int64_t B, int64_t N, int64_t K, int bits);
+
 /*
  * Quantise fp32 weights W[N][K] (device) to packed codes (device) with a
  * codebook built for (bits, base, range, flags) -- Eq. (1) with the
@@ -165,7 +175,10 @@ logq_status logq_quantize(const float* W, int64_t N, int64_t K, int bits, double
  *   rounded to nearest-even.  All device pointers 16-byte aligned.
  *   B <= 16 (4-bit) or B <= 4 (3- and 8-bit) runs the decode GEMV /
  *   skinny-GEMM kernel on CUDA cores; larger B runs the prefill GEMM kernel
- *   on the tensor cores (tcgen05).
+ *   on the tensor cores (tcgen05), as do 4-bit batches of 8..16 when the
+ *   workspace (see logq_linear_workspace_bytes) lets that launch keep at
+ *   least half of the SMs busy.  Calls sharing a workspace must be ordered
+ *   on one stream (partial sums may live in it).
  * Asynchronous.  Errors: LOGQ_ERR_INVALID_ARG, LOGQ_ERR_UNSUPPORTED,
  * LOGQ_ERR_WORKSPACE, LOGQ_ERR_CUDA (launch).  A device-side wait that hit
  * its bound is reported later by logq_workspace_status. */

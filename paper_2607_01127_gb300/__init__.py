@@ -37,7 +37,8 @@ LOGQ_ERR_NOT_PD = 7
 LOGQ_F32, LOGQ_BF16, LOGQ_F16 = 0, 1, 2
 LOGQ_SHIFT_EXACT, LOGQ_SHIFT_FLOOR = 0, 1
 
-EXPORTED = ("logq_build_codebook", "logq_packed_bytes", "logq_workspace_bytes", "logq_quantize",
+EXPORTED = ("logq_build_codebook", "logq_packed_bytes", "logq_workspace_bytes", "logq_linear_workspace_bytes",
+            "logq_quantize",
             "logq_linear", "logq_workspace_status", "logq_status_string", "logq_device_sm_count",
             "logq_quantize_noalloc", "logq_linear_grouped", "logq_energy_scratch_bytes",
             "logq_quantize_energy", "logq_gptq_factor_scratch_bytes", "logq_gptq_factor",
@@ -88,6 +89,8 @@ def _load() -> ctypes.CDLL:
     lib.logq_packed_bytes.restype = ctypes.c_size_t
     lib.logq_workspace_bytes.argtypes = []
     lib.logq_workspace_bytes.restype = ctypes.c_size_t
+    lib.logq_linear_workspace_bytes.argtypes = [c_i64, c_i64, c_i64, c_int]
+    lib.logq_linear_workspace_bytes.restype = ctypes.c_size_t
     lib.logq_quantize.argtypes = [P, c_i64, c_i64, c_int, c_dbl, c_dbl, c_int, P,
                                   ctypes.POINTER(Codebook), P, ctypes.c_size_t, P]
     lib.logq_quantize.restype = c_int
@@ -182,10 +185,17 @@ def logq_workspace_bytes() -> int:
     return int(_lib().logq_workspace_bytes())
 
 
-def new_workspace(device=None):
-    """Zero-filled device workspace of logq_workspace_bytes() bytes."""
+def logq_linear_workspace_bytes(B: int, N: int, K: int, bits: int) -> int:
+    return int(_lib().logq_linear_workspace_bytes(int(B), int(N), int(K), int(bits)))
+
+
+def new_workspace(device=None, nbytes: int | None = None):
+    """Zero-filled device workspace: logq_workspace_bytes() bytes, or nbytes (at
+    least that) -- e.g. the largest logq_linear_workspace_bytes() of the
+    products it will serve, so that tensor-core launches may split k ranges."""
     import torch
-    return torch.zeros(logq_workspace_bytes(), dtype=torch.uint8, device=device or "cuda")
+    n = logq_workspace_bytes() if nbytes is None else max(int(nbytes), logq_workspace_bytes())
+    return torch.zeros(n, dtype=torch.uint8, device=device or "cuda")
 
 
 def logq_quantize(W, bits: int, base: float, range_: float = 0.0, flags: int = LOGQ_SHIFT_EXACT,
@@ -310,7 +320,7 @@ def logq_linear(codes, cb: Codebook, X, N: int, K: int, y_dtype=None, Y=None, wo
     assert Y.dtype == _torch_dtype(yd) and Y.is_contiguous() and Y.numel() == B * N, \
         "Y must be a contiguous [B, N] tensor of the output dtype"
     if workspace is None:
-        workspace = new_workspace(X.device)
+        workspace = new_workspace(X.device, logq_linear_workspace_bytes(B, N, K, cb.bits))
     st = _lib().logq_linear(ctypes.c_void_p(codes.data_ptr()), ctypes.byref(cb), ctypes.c_void_p(X.data_ptr()),
                          xd, B, int(N), int(K), ctypes.c_void_p(Y.data_ptr()), yd,
                          ctypes.c_void_p(workspace.data_ptr()), workspace.numel(), _stream_ptr(stream))

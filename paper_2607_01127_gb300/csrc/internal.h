@@ -54,6 +54,7 @@ struct LinearArgs {
     int y_dtype;            // logq_dtype of Y
     uint16_t lvl16[256];    // code-indexed 16-bit levels in X's dtype (2^bits used)
     Workspace* ws;
+    size_t ws_bytes;        // the caller's workspace bytes (beyond kWorkspaceBytes: split-k partial sums)
 };
 
 // A grouped decode launch: up to four matrices that share X (e.g. q/k/v or
@@ -114,6 +115,17 @@ cudaError_t launch_gptq_factor(const float* H, int64_t K, double damp, float* U,
                                uint32_t* not_pd, cudaStream_t s);
 cudaError_t launch_gemv_group(const GroupArgs& a, cudaStream_t s);
 cudaError_t launch_prefill(const LinearArgs& a, cudaStream_t s);
+// Tensor-core launch plan of a B x N x K product: token-tile width, k ranges per
+// output tile (the partial sums need part_bytes of workspace beyond
+// kWorkspaceBytes; at most part_bytes_avail are used).
+struct PrefillPlan {
+    int bn;
+    int splits;
+    int ksplit;
+    size_t part_bytes;
+    double est_us;          // estimated launch time on a GB300 (planning only)
+};
+PrefillPlan prefill_plan(int64_t B, int64_t N, int64_t K, size_t part_bytes_avail);
 bool gemv_supports(int bits, int64_t B);
 
 }  // namespace logq

@@ -137,6 +137,33 @@ uint16_t f16_bits_of(float v)
 
 logq_status cuda_status(cudaError_t e) { return e == cudaSuccess ? LOGQ_OK : LOGQ_ERR_CUDA; }
 
+// 4-bit batches from this size up to 16 may run on the tensor cores instead of
+// the CUDA-core skinny GEMM (whose fp32 FMAs bound it at 16 per weight).
+#ifndef LOGQ_TC_MIN_BATCH
+#define LOGQ_TC_MIN_BATCH 8
+#endif
+
+// Batches that always run on the tensor cores, or may (4-bit, LOGQ_TC_MIN_BATCH..16).
+bool tensor_core_batch(int bits, int64_t B)
+{
+    return !gemv_supports(bits, B) || (bits == 4 && B >= LOGQ_TC_MIN_BATCH && B <= 16);
+}
+
+// A 4-bit batch of LOGQ_TC_MIN_BATCH..16 takes the tensor cores when their
+// estimated time beats the CUDA-core kernel's: ~27 us per 58.7 M weights at
+// batches up to 8 and ~49 us at 9..16 (the batch is padded to 8 or 16; fp32
+// FMAs bound it), plus ~2 us per launch (measured on the GB300 on the
+// Llama-3.1-8B shapes).  The tensor-core estimate depends on how far the caller's
+// workspace lets the k ranges split (prefill_plan).
+bool use_small_batch_tc(int bits, int64_t B, int64_t N, int64_t K, size_t workspace_bytes)
+{
+    if (!(bits == 4 && B >= LOGQ_TC_MIN_BATCH && B <= 16)) return false;
+    const size_t avail = workspace_bytes > kWorkspaceBytes ? workspace_bytes - kWorkspaceBytes : 0;
+    const PrefillPlan pl = prefill_plan(B, N, K, avail);
+    const double cuda_us = (double)N * (double)K * (B <= 8 ? 0.46e-6 : 0.84e-6) + 2.0;
+    return pl.est_us < cuda_us;
+}
+
 }  // namespace
 
 extern "C" {
@@ -203,6 +230,14 @@ size_t logq_packed_bytes(int64_t N, int64_t K, int bits)
 }
 
 size_t logq_workspace_bytes(void) { return kWorkspaceBytes; }
+
+size_t logq_linear_workspace_bytes(int64_t B, int64_t N, int64_t K, int bits)
+{
+    if (B <= 0 || logq_packed_bytes(N, K, bits) == 0) return 0;
+    if (!tensor_core_batch(bits, B)) return kWorkspaceBytes;
+    if (gemv_supports(bits, B) && !use_small_batch_tc(bits, B, N, K, (size_t)-1)) return kWorkspaceBytes;
+    return kWorkspaceBytes + prefill_plan(B, N, K, (size_t)-1).part_bytes;
+}
 
 logq_status logq_quantize(const float* W, int64_t N, int64_t K, int bits, double base,
                           double range, int flags, uint8_t* codes, logq_codebook* cb_out,
@@ -340,9 +375,11 @@ logq_status logq_linear(const uint8_t* codes, const logq_codebook* cb, const voi
     const uint16_t* tab = a.x_f16 ? cb->level_f16 : cb->level_bf16;
     for (int c = 0; c < (1 << cb->bits); ++c) a.lvl16[c] = tab[c];
     a.ws = static_cast<Workspace*>(workspace);
+    a.ws_bytes = workspace_bytes;
 
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    if (gemv_supports(cb->bits, B)) return cuda_status(launch_gemv(a, s));
+    if (gemv_supports(cb->bits, B) && !use_small_batch_tc(cb->bits, B, N, K, workspace_bytes))
+        return cuda_status(launch_gemv(a, s));
     const cudaError_t e = launch_prefill(a, s);
     if (e == cudaErrorNotSupported) return LOGQ_ERR_UNSUPPORTED;
     return cuda_status(e);
@@ -371,7 +408,9 @@ logq_status logq_linear_grouped(const logq_linear_item* items, int count, const 
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     Workspace* ws = static_cast<Workspace*>(workspace);
     const int x_f16 = (x_dtype == LOGQ_F16);
-    if (gemv_supports(bits, B)) {
+    bool all_tc = true;                     // every item takes the small-batch tensor-core path
+    for (int i = 0; i < count; ++i) all_tc = all_tc && use_small_batch_tc(bits, B, items[i].N, K, workspace_bytes);
+    if (gemv_supports(bits, B) && !all_tc) {
         GroupArgs g;
         memset(&g, 0, sizeof g);
         g.count = count;

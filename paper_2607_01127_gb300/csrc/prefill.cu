@@ -3,7 +3,11 @@
 // LUT reads, so here each weight is dequantised once per tile and reused by a
 // dense bf16/fp16 contraction).
 //
-// One persistent CTA per SM walks 128 (weights) x 256 (tokens) output tiles.
+// One persistent CTA per SM walks 128 (weights) x BN (tokens) output tiles, BN
+// = 256 for prefill and 16 for small batches; where there are too few tiles
+// to fill the SMs, each tile's k range is split into ranges taken by
+// different CTAs, which write fp32 partial sums to the caller's workspace and
+// a second kernel adds them in a fixed order.
 // The dequantised weight tile (the MMA's A operand) lives in tensor memory, not
 // in shared memory: tensor memory holds one fp32 accumulator (256 columns) and
 // eight weight stages (32 columns each), and shared memory holds the pair table
@@ -48,7 +52,7 @@ namespace logq {
 namespace {
 
 constexpr int kBM = 128;                 // weight rows per tile (MMA M)
-constexpr int kBN = 256;                 // tokens per tile (MMA N)
+constexpr int kBNMax = 256;              // widest token tile (MMA N)
 constexpr int kBK = 64;                  // k per stage (one 128-byte swizzle atom of bf16)
 constexpr int kXStages = 5;              // X tiles in flight (TMA)
 constexpr int kWStages = 8;              // dequantised weight tiles in flight (tensor memory)
@@ -58,7 +62,6 @@ constexpr int kDecodeThreads = 32 * kDecodeWarps;  // two threads per weight row
 constexpr int kEpiWarps = 8;                       // two per TMEM lane quarter
 constexpr int kEpi0 = 2, kDec0 = kEpi0 + kEpiWarps;  // first epilogue / decode warp
 constexpr int kThreads = 32 * (kDec0 + kDecodeWarps);  // producer, MMA, epilogue, decode
-constexpr int kXStageBytes = kBN * kBK * 2;      // 32 KiB
 constexpr int kCodeSlotBytes = 16;               // codes of half a row and stage (<= 16 B)
 constexpr int kCodeStageBytes = kDecodeThreads * kCodeSlotBytes;
 // Shared address at which dynamic shared memory starts in a kernel without
@@ -67,7 +70,7 @@ constexpr uint32_t kTabOff = 1024;
 constexpr uint32_t kTabRow = 256;                // 32 lane copies in the first 128 bytes
 constexpr uint32_t kTabRegion = 256 * kTabRow;   // table rows (the 4-bit table uses all 256)
 constexpr uint32_t kTmemCols = 512;              // accumulator (256) + weight stages (8 x 32)
-constexpr uint32_t kWCol0 = kBN;                 // first column of weight stage 0
+constexpr uint32_t kWCol0 = kBNMax;              // first column of weight stage 0 (after the widest accumulator)
 constexpr uint32_t kWStageCols = kBK / 2;        // 64 k of 16-bit values = 32 columns
 static_assert(kWCol0 + kWStages * kWStageCols <= kTmemCols, "weight stages must fit in tensor memory");
 constexpr long long kWaitLimit = 2000000000LL;   // cycles (~1 s)
@@ -83,12 +86,15 @@ struct PrefillParams {
     const uint8_t* codes;
     void* Y;
     Workspace* ws;
+    float* part;            // splits > 1: fp32 partial sums [splits][B][N] (caller's workspace)
     int64_t N;
     int32_t K, B;
     int64_t row_bytes;
     int32_t bits;
     int32_t y_dtype;
     int32_t n_tiles_n, n_tiles_t;
+    int32_t splits;         // k ranges per output tile
+    int32_t ksplit;         // k-steps per range (the last may be shorter)
     uint32_t idesc;
     uint32_t smem_bytes;    // dynamic shared memory of the launch (layout check)
     uint16_t lvl16[256];    // code-indexed 16-bit levels (2^bits used)
@@ -294,10 +300,13 @@ __device__ __forceinline__ void sts128(uint32_t addr, uint32_t a, uint32_t b, ui
 // (two ring slots), each byte resolves to one value (the table holds it in
 // both halves) and two values form a pair with one byte permute; the deeper
 // code footprint leaves room for RING = 3 stages in the table rows' halves.
-template <bool EIGHT>
+template <bool EIGHT, int BN>
 __global__ void __launch_bounds__(kThreads, 1)
 prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ CUtensorMap xmap)
 {
+    static_assert(BN >= 16 && BN <= kBNMax && BN % 16 == 0, "MMA N with M = 128");
+    constexpr int XB = BN * kBK * 2;                     // bytes of one X stage
+    constexpr int kChunks = ((BN < 128 ? BN : 128) + 31) / 32;   // 32-column drains per epilogue warp
     constexpr int SLOTS = EIGHT ? 2 : 1;                 // 16-byte ring slots per thread and stage
     constexpr int RING = EIGHT ? 3 : kCodeRing;          // code stages in flight per decode thread
     static_assert(RING * SLOTS * kCodeStageBytes <= 256 * 128, "code ring must fit in the table rows' free halves");
@@ -305,7 +314,7 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
     // Layout: pair table (code ring in its rows' free halves) | X stages | barriers
     const uint32_t sbase = smem_u32(smem_raw);
     const uint32_t xs0 = sbase + kTabRegion;
-    const uint32_t bar0 = xs0 + kXStages * kXStageBytes;
+    const uint32_t bar0 = xs0 + kXStages * XB;
     const uint32_t layout_end = bar0 + 256;
     // the lookups address the table as an offset from kTabOff; refuse a launch
     // whose shared window differs or is too small for this layout
@@ -382,7 +391,16 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
     const uint32_t tmem_base = *reinterpret_cast<volatile uint32_t*>(gen + tmem_slot);
 
     const int ksteps = p.K / kBK;
-    const int ntiles = p.n_tiles_n * p.n_tiles_t;
+    const int ntiles = p.n_tiles_n * p.n_tiles_t * p.splits;
+    // tile -> (weight-row tile, token tile, k range); the weight-row tile varies fastest
+    auto tile_n = [&](int tile) { return tile % p.n_tiles_n; };
+    auto tile_t = [&](int tile) { return (tile / p.n_tiles_n) % p.n_tiles_t; };
+    auto tile_sp = [&](int tile) { return tile / (p.n_tiles_n * p.n_tiles_t); };
+    auto k_begin = [&](int tile) { return tile_sp(tile) * p.ksplit; };
+    auto k_end = [&](int tile) {
+        const int e = (tile_sp(tile) + 1) * p.ksplit;
+        return e < ksteps ? e : ksteps;
+    };
 
     if (warp == 0) {
         // ---------------- TMA producer ----------------
@@ -395,28 +413,42 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         // tile ahead so the decode warps' copies hit L2
         auto prefetch_codes = [&](int tile) {
             if (tile >= ntiles) return;
-            const int64_t n0 = (int64_t)(tile % p.n_tiles_n) * kBM;
+            const int64_t n0 = (int64_t)tile_n(tile) * kBM;
             const int64_t rows = (p.N - n0) < kBM ? (p.N - n0) : kBM;
             const uint8_t* base = p.codes + n0 * p.row_bytes;
-            const int64_t bytes = rows * p.row_bytes;
-            for (int64_t off = (int64_t)lane * 16384; off < bytes; off += 32 * 16384) {
-                const int64_t nb = (bytes - off) < 16384 ? (bytes - off) : 16384;
-                asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base + off), "r"((uint32_t)nb)
-                             : "memory");
+            if (p.splits == 1) {
+                const int64_t bytes = rows * p.row_bytes;
+                for (int64_t off = (int64_t)lane * 16384; off < bytes; off += 32 * 16384) {
+                    const int64_t nb = (bytes - off) < 16384 ? (bytes - off) : 16384;
+                    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base + off), "r"((uint32_t)nb)
+                                 : "memory");
+                }
+                return;
             }
+            // the tile's k range of each row, widened to 16-byte bounds inside the row
+            // (row_bytes is a multiple of 16, and of the k-step count)
+            const int64_t step_bytes = p.row_bytes / ksteps;
+            const int64_t b0 = ((int64_t)k_begin(tile) * step_bytes) & ~(int64_t)15;
+            int64_t b1 = ((int64_t)k_end(tile) * step_bytes + 15) & ~(int64_t)15;
+            if (b1 > p.row_bytes) b1 = p.row_bytes;
+            for (int64_t r = lane; r < rows; r += 32)
+                asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base + r * p.row_bytes + b0),
+                             "r"((uint32_t)(b1 - b0))
+                             : "memory");
         };
         prefetch_codes(blockIdx.x);
         for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
-            const int t0 = (tile / p.n_tiles_n) * kBN;
+            const int t0 = tile_t(tile) * BN;
             prefetch_codes(tile + gridDim.x);
-            for (int ks = 0; ks < ksteps; ++ks) {
+            const int kb = k_begin(tile), ke = k_end(tile);
+            for (int ks = kb; ks < ke; ++ks) {
                 if (!warp_wait(xempty(stage), phase ^ 1u, abort_flag, p.ws, kWaitProducer)) {
                     ok = false;
                     break;
                 }
                 if (elect_one()) {
-                    mbar_expect_tx(xfull(stage), kXStageBytes);
-                    tma_load_2d(xs0 + stage * kXStageBytes, &xmap, ks * kBK, t0, xfull(stage));
+                    mbar_expect_tx(xfull(stage), XB);
+                    tma_load_2d(xs0 + stage * XB, &xmap, ks * kBK, t0, xfull(stage));
                 }
                 __syncwarp();
                 issued |= 1u << stage;
@@ -451,7 +483,8 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
             if (!warp_wait(accempty, ((uint32_t)it & 1u) ^ 1u, abort_flag, p.ws, kWaitMma)) break;
             tc_fence_after();
             const uint32_t dcol = tmem_base;
-            for (int ks = 0; ks < ksteps; ++ks) {
+            const int kb = k_begin(tile), ke = k_end(tile);
+            for (int ks = kb; ks < ke; ++ks) {
                 if (!warp_wait(xfull(xs), xph, abort_flag, p.ws, kWaitMma) ||
                     !warp_wait(wfull(wsg), wph, abort_flag, p.ws, kWaitMma)) {
                     ok = false;
@@ -459,13 +492,13 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
                 }
                 tc_fence_after();
                 const uint32_t acol = tmem_base + kWCol0 + (uint32_t)wsg * kWStageCols;
-                const uint64_t bdesc = smem_desc_sw128(xs0 + xs * kXStageBytes);
+                const uint64_t bdesc = smem_desc_sw128(xs0 + xs * XB);
                 if (elect_one()) {
 #pragma unroll
                     for (int kk = 0; kk < kBK / 16; ++kk) {
                         // 16 k: 8 columns of A further on; 32 bytes (2 descriptor units)
                         // further inside B's swizzle atom
-                        mma_f16_ta(dcol, acol + 8 * kk, bdesc + 2 * kk, p.idesc, (ks | kk) != 0);
+                        mma_f16_ta(dcol, acol + 8 * kk, bdesc + 2 * kk, p.idesc, (ks != kb) || kk != 0);
                     }
                     mma_commit(xempty(xs));
                     mma_commit(wempty(wsg));
@@ -492,17 +525,26 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
             if (!warp_wait(accfull, (uint32_t)it & 1u, abort_flag, p.ws, kWaitEpilogue)) break;
             tc_fence_after();
-            const int64_t n = (int64_t)(tile % p.n_tiles_n) * kBM + row;
-            const int tb0 = (tile / p.n_tiles_n) * kBN + ehalf * 128;
-            const int jmax = (p.B - tb0) < 128 ? (p.B - tb0) : 128;   // tokens of this half (may be <= 0)
-            if (p.y_dtype == LOGQ_F32) {
+            const int64_t n = (int64_t)tile_n(tile) * kBM + row;
+            const int tb0 = tile_t(tile) * BN + ehalf * 128;
+            // tokens of this half that exist (may be <= 0: the tile is narrower, or past B)
+            const int hcols = (BN - ehalf * 128) < 128 ? (BN - ehalf * 128) : 128;
+            const int jmax = (p.B - tb0) < hcols ? (p.B - tb0) : hcols;
+            if (hcols <= 0) {
+                // no column of this tile in this half: only hand the accumulator back
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(accempty);
+            } else if (p.splits > 1 || p.y_dtype == LOGQ_F32) {
+                // fp32 out: Y itself, or this k range's partial sums
+                float* yb = p.splits > 1 ? p.part + (int64_t)tile_sp(tile) * p.B * p.N : static_cast<float*>(p.Y);
 #pragma unroll 1
-                for (int c = 0; c < 4; ++c) {
+                for (int c = 0; c < kChunks; ++c) {
                     uint32_t v[32];
                     tmem_ld32(tq + (uint32_t)(c * 32), v);
                     const int jm = jmax - 32 * c;
                     if (n < p.N && jm > 0) {
-                        float* y = static_cast<float*>(p.Y) + (int64_t)(tb0 + 32 * c) * p.N + n;
+                        float* y = yb + (int64_t)(tb0 + 32 * c) * p.N + n;
 #pragma unroll
                         for (int j = 0; j < 32; ++j)
                             if (j < jm) y[(int64_t)j * p.N] = __uint_as_float(v[j]);
@@ -515,7 +557,7 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
                 const bool bf = p.y_dtype == LOGQ_BF16;
                 uint32_t pk[64];                        // tokens 2j, 2j+1 rounded to 16 bits
 #pragma unroll
-                for (int c = 0; c < 4; ++c) {
+                for (int c = 0; c < kChunks; ++c) {
                     uint32_t v[32];
                     tmem_ld32(tq + (uint32_t)(c * 32), v);
 #pragma unroll
@@ -566,24 +608,25 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         const int hbytes = EIGHT ? 32 : (p.bits == 4) ? 16 : 12;   // codes of one half row per stage
         int stage = 0;
         uint32_t phase = 0;
-        const int my_tiles = (ntiles > (int)blockIdx.x) ? (ntiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
-        const int total = my_tiles * ksteps;            // stages this CTA decodes
+        int total = 0;                                  // stages this CTA decodes
+        for (int t = (int)blockIdx.x; t < ntiles; t += (int)gridDim.x) total += k_end(t) - k_begin(t);
         // Cursor over (tile, k-step) advanced without divisions: one for the
         // copies issued ahead, one for the stage being decoded.
         struct Cursor {
-            int tile, ks;
+            int tile, ks, ke;                           // k-step and end of the tile's k range
             bool valid;                                 // this thread's row exists
             const uint8_t* row;                         // its codes, half h, stage 0
         };
         auto set_tile = [&](Cursor& c, int tile) {
             c.tile = tile;
-            c.ks = 0;
-            const int64_t n = (int64_t)(tile % p.n_tiles_n) * kBM + r;
+            c.ks = tile < ntiles ? k_begin(tile) : 0;
+            c.ke = tile < ntiles ? k_end(tile) : 0;
+            const int64_t n = (int64_t)tile_n(tile) * kBM + r;
             c.valid = tile < ntiles && n < p.N;
             c.row = p.codes + (c.valid ? n : 0) * p.row_bytes + (int64_t)h * hbytes;
         };
         auto step = [&](Cursor& c) {
-            if (++c.ks == ksteps) set_tile(c, c.tile + (int)gridDim.x);
+            if (++c.ks >= c.ke) set_tile(c, c.tile + (int)gridDim.x);
         };
         Cursor ahead, cur;
         set_tile(ahead, (int)blockIdx.x);
@@ -728,7 +771,7 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
     return fn;
 }
 
-uint32_t make_idesc(bool f16_inputs)
+uint32_t make_idesc(bool f16_inputs, int bn)
 {
     uint32_t d = 0;
     d |= 1u << 4;                                   // D format: fp32
@@ -736,17 +779,32 @@ uint32_t make_idesc(bool f16_inputs)
     d |= ab << 7;
     d |= ab << 10;
     // bits 15, 16: A and B K-major (0)
-    d |= (uint32_t)(kBN >> 3) << 17;                // N / 8
+    d |= (uint32_t)(bn >> 3) << 17;                 // N / 8
     d |= (uint32_t)(kBM >> 4) << 24;                // M / 16
     return d;
 }
 
 // Dynamic shared memory of the layout: table rows, X stages, barriers.
-constexpr uint32_t kSmemBytes = kTabRegion + kXStages * kXStageBytes + 256;
+constexpr uint32_t smem_bytes_for(int bn) { return kTabRegion + kXStages * (uint32_t)bn * kBK * 2 + 256; }
 
-template <bool EIGHT>
+// Fixed-order sum of the k ranges' fp32 partial sums: Y[i] = sum_s part[s][i]
+// (s = 0, 1, ...), rounded to Y's dtype.
+__global__ void __launch_bounds__(256) splitk_sum_kernel(const float* __restrict__ part, int splits, int64_t count,
+                                                         void* Y, int y_dtype)
+{
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < count; i += (int64_t)gridDim.x * blockDim.x) {
+        float v = part[i];
+        for (int sp = 1; sp < splits; ++sp) v += part[(int64_t)sp * count + i];
+        if (y_dtype == LOGQ_F32) static_cast<float*>(Y)[i] = v;
+        else if (y_dtype == LOGQ_BF16) static_cast<__nv_bfloat16*>(Y)[i] = __float2bfloat16_rn(v);
+        else static_cast<__half*>(Y)[i] = __float2half_rn(v);
+    }
+}
+
+template <bool EIGHT, int BN>
 cudaError_t launch(PrefillParams& p, const CUtensorMap& xmap, int grid, cudaStream_t s)
 {
+    constexpr uint32_t kSmemBytes = smem_bytes_for(BN);
     static uint32_t configured[64] = {0};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -758,16 +816,57 @@ cudaError_t launch(PrefillParams& p, const CUtensorMap& xmap, int grid, cudaStre
         if ((e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev)) != cudaSuccess) return e;
         const uint32_t bytes = kSmemBytes;
         if (reserved != (int)kTabOff || bytes > (uint32_t)optin) return cudaErrorNotSupported;
-        e = cudaFuncSetAttribute(prefill_kernel<EIGHT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+        e = cudaFuncSetAttribute(prefill_kernel<EIGHT, BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
         if (e != cudaSuccess) return e;
         configured[dev] = bytes;
     }
     p.smem_bytes = configured[dev];
-    prefill_kernel<EIGHT><<<grid, kThreads, configured[dev], s>>>(p, xmap);
+    prefill_kernel<EIGHT, BN><<<grid, kThreads, configured[dev], s>>>(p, xmap);
     return cudaGetLastError();
 }
 
 }  // namespace
+
+PrefillPlan prefill_plan(int64_t B, int64_t N, int64_t K, size_t part_bytes_avail)
+{
+    PrefillPlan pl;
+    pl.bn = B <= 16 ? 16 : kBNMax;
+    const int sms = sm_count() > 0 ? sm_count() : 148;
+    const int64_t tiles = ((N + kBM - 1) / kBM) * ((B + pl.bn - 1) / pl.bn);
+    const int64_t ksteps = K / kBK;
+    // Cost in k-step times (~0.5 us each on the GB300, for either tile width;
+    // the decode warps bound a stage): persistent CTAs take tiles in rounds,
+    // a tile of ks k-steps costing ks + 6 (pipeline fill, and the MMA waiting
+    // for the epilogue to drain the single accumulator).  A split adds the sum
+    // kernel (~6) and the partial sums' HBM traffic, written once and read once
+    // (8 bytes per output and range, at ~6 TB/s).  Each range keeps at least 8
+    // k-steps and the partials fit the caller's workspace.  (Fitted to launches
+    // of the Llama-3.1-8B shapes at batches 8-64 and 2048 tokens.)
+    auto cost = [&](int64_t splits, int64_t ksplit) {
+        const int64_t units = tiles * splits;
+        double c = (double)((units + sms - 1) / sms) * (double)(ksplit + 6);
+        if (splits > 1) c += 6.0 + (double)splits * (double)B * (double)N * 8.0 / 3.0e6;
+        return c;
+    };
+    pl.splits = 1;
+    pl.ksplit = (int)ksteps;
+    double best = cost(1, ksteps);
+    for (int64_t sp = 2; sp <= 32 && ksteps / sp >= 8; ++sp) {
+        const int64_t ksplit = (ksteps + sp - 1) / sp;
+        const int64_t real = (ksteps + ksplit - 1) / ksplit;       // ranges actually used
+        const size_t need = (size_t)real * (size_t)B * (size_t)N * 4;
+        if (need > part_bytes_avail) break;
+        const double c = cost(real, ksplit);
+        if (c < best) {
+            best = c;
+            pl.splits = (int)real;
+            pl.ksplit = (int)ksplit;
+        }
+    }
+    pl.part_bytes = pl.splits > 1 ? (size_t)pl.splits * (size_t)B * (size_t)N * 4 : 0;
+    pl.est_us = 0.5 * best + 3.0;
+    return pl;
+}
 
 cudaError_t launch_prefill(const LinearArgs& a, cudaStream_t s)
 {
@@ -777,7 +876,9 @@ cudaError_t launch_prefill(const LinearArgs& a, cudaStream_t s)
     memset(&xmap, 0, sizeof xmap);
     const cuuint64_t gdim[2] = {(cuuint64_t)a.K, (cuuint64_t)a.B};
     const cuuint64_t gstride[1] = {(cuuint64_t)a.K * 2};
-    const cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)kBN};
+    const size_t avail = a.ws_bytes > kWorkspaceBytes ? a.ws_bytes - kWorkspaceBytes : 0;
+    const PrefillPlan pl = prefill_plan(a.B, a.N, a.K, avail);
+    const cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)pl.bn};
     const cuuint32_t estride[2] = {1, 1};
     CUresult r = encode(&xmap, a.x_f16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
                         const_cast<void*>(a.X), gdim, gstride, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
@@ -797,14 +898,27 @@ cudaError_t launch_prefill(const LinearArgs& a, cudaStream_t s)
     p.row_bytes = (a.bits == 8) ? a.K : (a.bits == 4) ? a.K / 2 : a.K / 32 * 12;
     p.y_dtype = a.y_dtype;
     p.n_tiles_n = (int32_t)((a.N + kBM - 1) / kBM);
-    p.n_tiles_t = (int32_t)((a.B + kBN - 1) / kBN);
-    p.idesc = make_idesc(a.x_f16 != 0);
+    p.n_tiles_t = (int32_t)((a.B + pl.bn - 1) / pl.bn);
+    p.splits = pl.splits;
+    p.ksplit = pl.ksplit;
+    p.part = pl.splits > 1 ? reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(a.ws) + kWorkspaceBytes) : nullptr;
+    p.idesc = make_idesc(a.x_f16 != 0, pl.bn);
     for (int c = 0; c < (1 << a.bits); ++c) p.lvl16[c] = a.lvl16[c];
-    const int64_t ntiles = (int64_t)p.n_tiles_n * p.n_tiles_t;
+    const int64_t ntiles = (int64_t)p.n_tiles_n * p.n_tiles_t * p.splits;
     const int sms = sm_count() > 0 ? sm_count() : 148;
     const int grid = (int)(ntiles < sms ? ntiles : sms);
 
-    return a.bits == 8 ? launch<true>(p, xmap, grid, s) : launch<false>(p, xmap, grid, s);
+    cudaError_t e;
+    if (pl.bn == 16)
+        e = a.bits == 8 ? launch<true, 16>(p, xmap, grid, s) : launch<false, 16>(p, xmap, grid, s);
+    else
+        e = a.bits == 8 ? launch<true, kBNMax>(p, xmap, grid, s) : launch<false, kBNMax>(p, xmap, grid, s);
+    if (e != cudaSuccess || pl.splits == 1) return e;
+    const int64_t count = a.B * a.N;
+    int64_t blocks = (count + 255) / 256;
+    if (blocks > (int64_t)sms * 8) blocks = (int64_t)sms * 8;
+    splitk_sum_kernel<<<(int)blocks, 256, 0, s>>>(p.part, pl.splits, count, a.Y, a.y_dtype);
+    return cudaGetLastError();
 }
 
 }  // namespace logq

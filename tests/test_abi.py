@@ -95,6 +95,25 @@ def test_workspace_bytes(logq):
     assert logq.logq_workspace_bytes() == 256
 
 
+def test_linear_workspace_bytes(logq):
+    """4-bit products that stay on the CUDA cores need only the base workspace
+    (batches up to 7, and batches 8..16 where that kernel is estimated faster);
+    tensor-core products whose output tiles are too few to fill the GPU ask for
+    room for split-k partial sums (splits x B x N fp32); invalid sizes give 0."""
+    base = logq.logq_workspace_bytes()
+    assert logq.logq_linear_workspace_bytes(1, 4096, 4096, 4) == base
+    assert logq.logq_linear_workspace_bytes(4, 14336, 4096, 4) == base
+    assert logq.logq_linear_workspace_bytes(8, 4096, 14336, 4) == base
+    assert logq.logq_linear_workspace_bytes(16, 4096, 4096, 4) == base
+    for B, N, K, bits in [(16, 4096, 8192, 4), (16, 4096, 14336, 4), (64, 1024, 4096, 4), (12, 2048, 2048, 3)]:
+        extra = logq.logq_linear_workspace_bytes(B, N, K, bits) - base
+        assert extra > 0 and extra % (B * N * 4) == 0, (B, N, K, bits, extra)
+        splits = extra // (B * N * 4)
+        assert 2 <= splits <= K // 64 // 8
+    assert logq.logq_linear_workspace_bytes(0, 4096, 4096, 4) == 0
+    assert logq.logq_linear_workspace_bytes(16, 4096, 100, 4) == 0
+
+
 def test_status_strings(logq):
     for s in range(7):
         assert len(logq.status_string(s)) >= 2

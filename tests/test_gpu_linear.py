@@ -160,6 +160,54 @@ def test_prefill_bf16(logq, N, K, B, bits):
     run_case(logq, N, K, bits, B, torch.bfloat16, seed=N + B + bits)
 
 
+@pytest.mark.parametrize("N,K,B,ydt", [(4096, 8192, 16, torch.bfloat16), (4100, 8192, 12, None),
+                                       (4096, 14336, 16, torch.bfloat16), (4096, 8192, 9, torch.bfloat16)])
+def test_small_batch_tensor_cores_split_k(logq, N, K, B, ydt):
+    """4-bit batches of 9..16 on long-K shapes run on the tensor cores with each
+    output tile's k range split over CTAs (fp32 partials, fixed-order sum) when the
+    workspace has room; with the minimal workspace the same call keeps the
+    CUDA-core kernel.  Both match the oracle; base 3 makes almost every code
+    non-zero, so the two summation orders give different fp32 sums."""
+    codes, cb, ocb, q = make_layer(logq, N, K, 4, 3.0, N + B)
+    X = workloads.activations_torch(B, K, N + K, torch.bfloat16, "cuda")
+    wsb = logq.logq_linear_workspace_bytes(B, N, K, 4)
+    assert wsb > logq.logq_workspace_bytes()
+    Yt = logq.logq_linear(codes, cb, X, N, K, y_dtype=ydt, workspace=logq.new_workspace(nbytes=wsb))
+    Yc = logq.logq_linear(codes, cb, X, N, K, y_dtype=ydt, workspace=logq.new_workspace())
+    Yr, A = reference(X, q, ocb)
+    name = "f32" if ydt is None else "bf16"
+    check_linear(Yt.double().cpu().numpy(), Yr, A, name)
+    check_linear(Yc.double().cpu().numpy(), Yr, A, name)
+    assert not torch.equal(Yt, Yc)
+
+
+def test_small_batch_tensor_cores_without_split(logq):
+    """112 output tiles of 128 rows fill enough SMs without splitting the k range;
+    the tensor cores beat the CUDA-core kernel at batch 16 here, workspace or not."""
+    N, K, B = 14336, 2048, 16
+    assert logq.logq_linear_workspace_bytes(B, N, K, 4) == logq.logq_workspace_bytes()
+    codes, cb, ocb, q = make_layer(logq, N, K, 4, 3.0, 77)
+    X = workloads.activations_torch(B, K, 77, torch.bfloat16, "cuda")
+    Y = logq.logq_linear(codes, cb, X, N, K, y_dtype=torch.bfloat16, workspace=logq.new_workspace())
+    Yr, A = reference(X, q, ocb)
+    check_linear(Y.double().cpu().numpy(), Yr, A, "bf16")
+
+
+@pytest.mark.parametrize("bits,B", [(3, 8), (8, 16), (3, 5)])
+def test_small_batch_3_and_8_bit_on_tensor_cores(logq, bits, B):
+    """3- and 8-bit batches above 4 run on the tensor cores in 16-token tiles (split or not)."""
+    run_case(logq, 2048, 2048, bits, B, torch.bfloat16, ydt=torch.bfloat16, seed=bits * 10 + B,
+             base=1.25 if bits == 3 else 1.05)
+    run_case(logq, 300, 1152, bits, B, torch.bfloat16, seed=bits + B, base=1.25 if bits == 3 else 1.05)
+
+
+@pytest.mark.parametrize("N,K,B", [(1024, 4096, 64), (1000, 4096, 300), (200, 2048, 40)])
+def test_prefill_split_k(logq, N, K, B):
+    """Prefill shapes with too few output tiles split the k range (ragged N and B)."""
+    assert logq.logq_linear_workspace_bytes(B, N, K, 4) > logq.logq_workspace_bytes()
+    run_case(logq, N, K, 4, B, torch.bfloat16, ydt=torch.bfloat16, seed=N + B)
+
+
 @pytest.mark.parametrize("ydt", [torch.bfloat16, None])
 def test_prefill_output_dtypes_and_fp16(logq, ydt):
     run_case(logq, 512, 1024, 4, 256, torch.bfloat16, ydt=ydt, seed=5)
