@@ -56,13 +56,24 @@ constexpr int kBNMax = 256;              // widest token tile (MMA N)
 constexpr int kBK = 64;                  // k per stage (one 128-byte swizzle atom of bf16)
 constexpr int kXStages = 5;              // X tiles in flight (TMA)
 constexpr int kWStages = 8;              // dequantised weight tiles in flight (tensor memory)
-constexpr int kCodeRing = 7;             // code stages in flight per decode thread
-constexpr int kDecodeWarps = 8;
-constexpr int kDecodeThreads = 32 * kDecodeWarps;  // two threads per weight row
+// Decode warps: four per k slice of a stage (one per TMEM lane quarter), each
+// thread owning one weight row's kSliceK of the stage's 64 k.  Eight (two
+// slices of 32 k) measured faster than sixteen (four of 16 k, 72 registers):
+// the per-stage waits, tensor-memory store and arrive of each warp cost more
+// than the extra warps hide.
+#ifndef LOGQ_PREFILL_DECODE_WARPS
+#define LOGQ_PREFILL_DECODE_WARPS 8
+#endif
+constexpr int kDecodeWarps = LOGQ_PREFILL_DECODE_WARPS;
+static_assert(kDecodeWarps == 8 || kDecodeWarps == 16, "two or four k slices per stage");
+constexpr int kSlices = kDecodeWarps / 4;
+constexpr int kSliceK = 64 / kSlices;            // k per decode thread and stage: 32 or 16
+constexpr int kSlicePairs = kSliceK / 2;         // TMEM columns (16-bit pairs) per thread and stage
+constexpr int kDecodeThreads = 32 * kDecodeWarps;
 constexpr int kEpiWarps = 8;                       // two per TMEM lane quarter
 constexpr int kEpi0 = 2, kDec0 = kEpi0 + kEpiWarps;  // first epilogue / decode warp
 constexpr int kThreads = 32 * (kDec0 + kDecodeWarps);  // producer, MMA, epilogue, decode
-constexpr int kCodeSlotBytes = 16;               // codes of half a row and stage (<= 16 B)
+constexpr int kCodeSlotBytes = 16;               // ring slot: codes of one thread's slice (<= 16 B)
 constexpr int kCodeStageBytes = kDecodeThreads * kCodeSlotBytes;
 // Shared address at which dynamic shared memory starts in a kernel without
 // static shared memory (the per-CTA reserved area comes first).
@@ -194,6 +205,11 @@ __device__ __forceinline__ void cp_async_4(uint32_t dst, const void* src)
     asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(dst), "l"(src) : "memory");
 }
 
+__device__ __forceinline__ void cp_async_8(uint32_t dst, const void* src)
+{
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(dst), "l"(src) : "memory");
+}
+
 __device__ __forceinline__ void cp_async_16(uint32_t dst, const void* src)
 {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
@@ -233,13 +249,21 @@ __device__ __forceinline__ void mma_f16_ta(uint32_t tmem_d, uint32_t tmem_a, uin
 }
 
 // 16 consecutive columns of this warp's 32 TMEM lanes (lane i of the warp -> TMEM lane base + i).
-__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&v)[16])
+[[maybe_unused]] __device__ __forceinline__ void tmem_st_pairs(uint32_t taddr, const uint32_t (&v)[16])
 {
     asm volatile(
         "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
         "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};"
         ::"r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
           "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
+        : "memory");
+}
+
+[[maybe_unused]] __device__ __forceinline__ void tmem_st_pairs(uint32_t taddr, const uint32_t (&v)[8])
+{
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};"
+        ::"r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
         : "memory");
 }
 
@@ -296,10 +320,10 @@ __device__ __forceinline__ void sts128(uint32_t addr, uint32_t a, uint32_t b, ui
 
 // ------------------------------------------------------------------ kernel ---
 
-// EIGHT: 8-bit codes, one per byte: a thread's 32 k of a stage are 32 bytes
-// (two ring slots), each byte resolves to one value (the table holds it in
-// both halves) and two values form a pair with one byte permute; the deeper
-// code footprint leaves room for RING = 3 stages in the table rows' halves.
+// EIGHT: 8-bit codes, one per byte: a thread's kSliceK k of a stage are
+// kSliceK bytes (one or two ring slots), each byte resolves to one value (the
+// table holds it in both halves) and two values form a pair with one byte
+// permute.
 template <bool EIGHT, int BN>
 __global__ void __launch_bounds__(kThreads, 1)
 prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ CUtensorMap xmap)
@@ -307,8 +331,11 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
     static_assert(BN >= 16 && BN <= kBNMax && BN % 16 == 0, "MMA N with M = 128");
     constexpr int XB = BN * kBK * 2;                     // bytes of one X stage
     constexpr int kChunks = ((BN < 128 ? BN : 128) + 31) / 32;   // 32-column drains per epilogue warp
-    constexpr int SLOTS = EIGHT ? 2 : 1;                 // 16-byte ring slots per thread and stage
-    constexpr int RING = EIGHT ? 3 : kCodeRing;          // code stages in flight per decode thread
+    constexpr int SLOTS = (EIGHT && kSliceK == 32) ? 2 : 1;   // 16-byte ring slots per thread and stage
+    // code stages in flight per decode thread: as many as the free halves of the
+    // table rows hold, at most 7
+    constexpr int RING_FIT = (256 * 128) / (SLOTS * kCodeStageBytes);
+    constexpr int RING = RING_FIT < 7 ? RING_FIT : 7;
     static_assert(RING * SLOTS * kCodeStageBytes <= 256 * 128, "code ring must fit in the table rows' free halves");
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     // Layout: pair table (code ring in its rows' free halves) | X stages | barriers
@@ -599,13 +626,17 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         // ---------------- decode ----------------
         // tcgen05.st reaches only the warp's TMEM lane quarter (warp % 4), so the
         // weight row of a thread is its TMEM lane: row = 32 * (warp % 4) + lane.
+        // The warps of a quarter split the stage's 64 k into kSlices slices.
         const int dw = warp - kDec0;                    // 0 .. kDecodeWarps-1
         const int d = dw * 32 + lane;                   // code-ring slot, 0 .. kDecodeThreads-1
         const int r = (warp & 3) * 32 + lane;           // weight row within the tile
-        const int h = dw >> 2;                          // half: k 32h .. 32h+31 of the stage
-        const uint32_t tw = tmem_base + ((uint32_t)((warp & 3) * 32) << 16) + kWCol0 + (uint32_t)(16 * h);
+        const int h = dw >> 2;                          // slice: k kSliceK*h .. +kSliceK-1 of the stage
+        const uint32_t tw = tmem_base + ((uint32_t)((warp & 3) * 32) << 16) + kWCol0 + (uint32_t)(kSlicePairs * h);
         const uint32_t lane4 = 4u * (uint32_t)lane;
-        const int hbytes = EIGHT ? 32 : (p.bits == 4) ? 16 : 12;   // codes of one half row per stage
+        // bytes of one row's codes per stage, and where this thread's slice (for 3-bit:
+        // the 32-k group holding it) starts among them
+        const int step_bytes = EIGHT ? 64 : (p.bits == 4) ? 32 : 24;
+        const int slice_off = EIGHT ? kSliceK * h : (p.bits == 4) ? (kSliceK / 2) * h : 12 * ((kSliceK * h) / 32);
         int stage = 0;
         uint32_t phase = 0;
         int total = 0;                                  // stages this CTA decodes
@@ -615,7 +646,7 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         struct Cursor {
             int tile, ks, ke;                           // k-step and end of the tile's k range
             bool valid;                                 // this thread's row exists
-            const uint8_t* row;                         // its codes, half h, stage 0
+            const uint8_t* row;                         // its codes: slice, stage 0
         };
         auto set_tile = [&](Cursor& c, int tile) {
             c.tile = tile;
@@ -623,7 +654,7 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
             c.ke = tile < ntiles ? k_end(tile) : 0;
             const int64_t n = (int64_t)tile_n(tile) * kBM + r;
             c.valid = tile < ntiles && n < p.N;
-            c.row = p.codes + (c.valid ? n : 0) * p.row_bytes + (int64_t)h * hbytes;
+            c.row = p.codes + (c.valid ? n : 0) * p.row_bytes + slice_off;
         };
         auto step = [&](Cursor& c) {
             if (++c.ks >= c.ke) set_tile(c, c.tile + (int)gridDim.x);
@@ -633,13 +664,14 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         set_tile(cur, (int)blockIdx.x);
         auto issue = [&](int g) {
             if (g < total && ahead.valid) {
-                const uint8_t* src = ahead.row + (int64_t)ahead.ks * (2 * hbytes);
+                const uint8_t* src = ahead.row + (int64_t)ahead.ks * step_bytes;
                 const uint32_t dst = ring_slot(g % RING, SLOTS * d);
                 if constexpr (EIGHT) {
                     cp_async_16(dst, src);
-                    cp_async_16(dst + 16, src + 16);
+                    if constexpr (kSliceK == 32) cp_async_16(dst + 16, src + 16);
                 } else if (p.bits == 4) {
-                    cp_async_16(dst, src);
+                    if constexpr (kSliceK == 32) cp_async_16(dst, src);
+                    else cp_async_8(dst, src);
                 } else {
                     cp_async_4(dst, src);
                     cp_async_4(dst + 4, src + 4);
@@ -649,18 +681,22 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
             if (g < total) step(ahead);
             cp_async_commit();
         };
-        // Resolve the codes of one stage (its slot in the ring) into 16 pair values.
-        auto resolve = [&](int slot, bool valid, uint32_t (&pr)[16]) {
+        // Resolve the codes of one stage (its slot in the ring) into the slice's pair values.
+        auto resolve = [&](int slot, bool valid, uint32_t (&pr)[kSlicePairs]) {
             if constexpr (EIGHT) {
-                // word i holds the codes of k = 32h + 4i .. +3: pairs 2i and 2i + 1
-                uint4 c0 = make_uint4(0, 0, 0, 0), c1 = make_uint4(0, 0, 0, 0);
+                // word i holds the codes of k = kSliceK h + 4i .. +3: pairs 2i and 2i + 1
+                constexpr int NWD = kSliceK / 4;
+                uint32_t cw8[8] = {0, 0, 0, 0, 0, 0, 0, 0};
                 if (valid) {
-                    c0 = lds128(ring_slot(slot, SLOTS * d));
-                    c1 = lds128(ring_slot(slot, SLOTS * d) + 16);
+                    const uint4 c0 = lds128(ring_slot(slot, SLOTS * d));
+                    cw8[0] = c0.x; cw8[1] = c0.y; cw8[2] = c0.z; cw8[3] = c0.w;
+                    if constexpr (NWD == 8) {
+                        const uint4 c1 = lds128(ring_slot(slot, SLOTS * d) + 16);
+                        cw8[4] = c1.x; cw8[5] = c1.y; cw8[6] = c1.z; cw8[7] = c1.w;
+                    }
                 }
-                const uint32_t cw8[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {
+                for (int i = 0; i < NWD; ++i) {
                     const uint32_t v0 = lds_tab(prmt(cw8[i], lane4, 0x7604u));
                     const uint32_t v1 = lds_tab(prmt(cw8[i], lane4, 0x7614u));
                     const uint32_t v2 = lds_tab(prmt(cw8[i], lane4, 0x7624u));
@@ -674,9 +710,9 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
             if (valid) cv = lds128(ring_slot(slot, d));
             const uint32_t cw[4] = {cv.x, cv.y, cv.z, cv.w};
             if (p.bits == 4) {
-                // word i holds k = 32h + 8i .. +7 -> 16-byte chunk 4h + i of the row
+                // word i holds k = kSliceK h + 8i .. +7
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
+                for (int i = 0; i < kSliceK / 8; ++i) {
                     const uint32_t c = cw[i];
                     pr[4 * i + 0] = lds_tab(prmt(c, lane4, 0x7604u));
                     pr[4 * i + 1] = lds_tab(prmt(c, lane4, 0x7614u));
@@ -684,22 +720,36 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
                     pr[4 * i + 3] = lds_tab(prmt(c, lane4, 0x7634u));
                 }
             } else {
-                // one 12-byte group of 32 k; pair p -> chunk 4h + p / 4
+                // one 12-byte group of 32 k: pair q (k 2q, 2q + 1) is the 6-bit field q % 5
+                // of word q / 5 (q < 15); pair 15 takes the two top bits of each word
+                auto pair_off = [&](int q) -> uint32_t {
+                    if (q == 15)
+                        return ((cw[0] >> 22) & 0x0300u) | ((cw[1] >> 20) & 0x0c00u) | ((cw[2] >> 18) & 0x3000u) | lane4;
+                    const int f = q % 5;
+                    const uint32_t x = cw[q / 5];
+                    const uint32_t field = f == 0 ? (x << 8) : f == 1 ? (x << 2) : f == 2 ? (x >> 4)
+                                         : f == 3 ? (x >> 10) : (x >> 16);
+                    return (field & 0x3f00u) | lane4;
+                };
+                if constexpr (kSliceK == 32) {
 #pragma unroll
-                for (int i = 0; i < 3; ++i) {
-                    pr[5 * i + 0] = lds_tab(((cw[i] << 8) & 0x3f00u) | lane4);
-                    pr[5 * i + 1] = lds_tab(((cw[i] << 2) & 0x3f00u) | lane4);
-                    pr[5 * i + 2] = lds_tab(((cw[i] >> 4) & 0x3f00u) | lane4);
-                    pr[5 * i + 3] = lds_tab(((cw[i] >> 10) & 0x3f00u) | lane4);
-                    pr[5 * i + 4] = lds_tab(((cw[i] >> 16) & 0x3f00u) | lane4);
+                    for (int q = 0; q < 16; ++q) pr[q] = lds_tab(pair_off(q));
+                } else {
+                    // this slice is half of the group: pairs 8 (h & 1) .. +7
+                    if ((h & 1) == 0) {
+#pragma unroll
+                        for (int q = 0; q < 8; ++q) pr[q] = lds_tab(pair_off(q));
+                    } else {
+#pragma unroll
+                        for (int q = 0; q < 8; ++q) pr[q] = lds_tab(pair_off(8 + q));
+                    }
                 }
-                pr[15] = lds_tab(((cw[0] >> 22) & 0x0300u) | ((cw[1] >> 20) & 0x0c00u) | ((cw[2] >> 18) & 0x3000u) | lane4);
             }
         };
         // Software pipeline: the pairs of stage g+1 are looked up while stage g
         // waits for its weight slot and is stored.
         for (int g = 0; g < RING - 1; ++g) issue(g);
-        uint32_t pr_a[16], pr_b[16];
+        uint32_t pr_a[kSlicePairs], pr_b[kSlicePairs];
         int slot = 0;                                   // ring slot of stage g
         if (total > 0) {
             issue(RING - 1);
@@ -711,7 +761,7 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         // stage's (cur) once its weight slot is free.  Called with the two
         // buffers in alternating roles, so no pairs are copied.
         bool ok = true;
-        auto stage_step = [&](int g, const uint32_t (&cur_pr)[16], uint32_t (&nxt_pr)[16]) {
+        auto stage_step = [&](int g, const uint32_t (&cur_pr)[kSlicePairs], uint32_t (&nxt_pr)[kSlicePairs]) {
             if (++slot == RING) slot = 0;
             if (g + 1 < total) {
                 issue(g + RING);
@@ -724,8 +774,8 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
                 return;
             }
             tc_fence_after();
-            // pair q holds k = 32h + 2q (low half) and 32h + 2q + 1: column 16h + q of the stage
-            tmem_st16(tw + (uint32_t)stage * kWStageCols, cur_pr);
+            // pair q holds k = kSliceK h + 2q (low half) and + 1: column kSlicePairs h + q of the stage
+            tmem_st_pairs(tw + (uint32_t)stage * kWStageCols, cur_pr);
             tmem_wait_st();
             tc_fence_before();            // this warp's tensor-memory writes -> the MMA issuer
             __syncwarp();
