@@ -429,6 +429,7 @@ def time_prefill(logq, torch, dev, reps: int = 3):
     # room for split-k partial sums of every shape (k/v: too few output tiles to fill the GPU)
     ws = logq.new_workspace(dev, max(logq.logq_linear_workspace_bytes(PREFILL_TOKENS, N, K, 4)
                                      for N, K in workloads.LLAMA_8B_SHAPES.values()))
+    s = torch.cuda.Stream(dev)
     tot_flop, tot_t = 0.0, 0.0
     for pi, name in enumerate(workloads.PROJ_NAMES):
         if name in ("v", "up"):
@@ -440,19 +441,23 @@ def time_prefill(logq, torch, dev, reps: int = 3):
         X = workloads.activations_torch(PREFILL_TOKENS, K, pi, torch.bfloat16, dev)
         Y = torch.empty(PREFILL_TOKENS, N, dtype=torch.bfloat16, device=dev)
         try:
-            logq.logq_linear(codes, cb, X, N, K, y_dtype=torch.bfloat16, Y=Y, workspace=ws)
+            logq.logq_linear(codes, cb, X, N, K, y_dtype=torch.bfloat16, Y=Y, workspace=ws, stream=s)
         except logq.LogqError as e:
             if e.status == logq.LOGQ_ERR_UNSUPPORTED:
                 return None
             raise
         torch.cuda.synchronize()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record()
-        for _ in range(reps):
-            logq.logq_linear(codes, cb, X, N, K, y_dtype=torch.bfloat16, Y=Y, workspace=ws)
-        e1.record()
+        # reps back-to-back calls captured in a graph (a split call is two launches:
+        # the GEMM and the sum of its k ranges), so host launch gaps stay out
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(s):
+            with torch.cuda.graph(g, stream=s):
+                for _ in range(reps):
+                    logq.logq_linear(codes, cb, X, N, K, y_dtype=torch.bfloat16, Y=Y, workspace=ws, stream=s)
+        g.replay()
         torch.cuda.synchronize()
-        t = e0.elapsed_time(e1) / reps * 1e-3
+        t = time_replays(torch, g, s, 2) / (2 * reps)
+        del g
         flop = 2.0 * PREFILL_TOKENS * N * K
         res[name] = {"N": N, "K": K, "us": round(t * 1e6, 2), "tflops": round(flop / t / 1e12, 1)}
         tot_flop += flop * (2 if name in ("k", "gate") else 1)
