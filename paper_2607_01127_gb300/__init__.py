@@ -351,7 +351,8 @@ def logq_linear_grouped(items, X, K: int, y_dtype=None, workspace=None, prefetch
         arr[i] = LinearItem(ctypes.c_void_p(codes.data_ptr()), ctypes.pointer(cb), int(N),
                             ctypes.c_void_p(Y.data_ptr()))
     if workspace is None:
-        workspace = new_workspace(X.device)
+        workspace = new_workspace(X.device, max(logq_linear_workspace_bytes(B, int(N), K, cb.bits)
+                                                for _, cb, N, _ in items))
     pf_ptr = ctypes.c_void_p(prefetch.data_ptr()) if prefetch is not None else None
     pf_bytes = int(prefetch_bytes) if prefetch is not None else 0
     st = _lib().logq_linear_grouped(arr, len(items), ctypes.c_void_p(X.data_ptr()), xd, B, int(K), yd, pf_ptr,

@@ -208,6 +208,35 @@ def test_prefill_split_k(logq, N, K, B):
     run_case(logq, N, K, 4, B, torch.bfloat16, ydt=torch.bfloat16, seed=N + B)
 
 
+@pytest.mark.parametrize("bits,N,K,B,xdt", [(4, 1024, 4096, 64, torch.float16), (3, 1000, 2048, 40, torch.bfloat16),
+                                            (8, 1024, 4096, 48, torch.bfloat16)])
+def test_prefill_split_k_dtypes(logq, bits, N, K, B, xdt):
+    """Split k ranges with fp16 activations and output, 3-bit groups and 8-bit codes."""
+    assert logq.logq_linear_workspace_bytes(B, N, K, bits) > logq.logq_workspace_bytes()
+    run_case(logq, N, K, bits, B, xdt, ydt=xdt, seed=N + B + bits, base=1.25 if bits == 3 else 1.5)
+
+
+def test_grouped_split_k_equals_single_calls(logq):
+    """A grouped call at batch 64 runs each matrix on the tensor cores with its k range
+    split, one after another through the same workspace: each output equals the single
+    call's bit for bit and matches the oracle."""
+    K, B = 4096, 64
+    shapes = [(1024, 1.4), (512, 1.7), (512, 2.0)]
+    layers = [make_layer(logq, N, K, 4, base, seed=90 + i) for i, (N, base) in enumerate(shapes)]
+    X = workloads.activations_torch(B, K, 91, torch.bfloat16, "cuda")
+    wsb = max(logq.logq_linear_workspace_bytes(B, N, K, 4) for N, _ in shapes)
+    assert wsb > logq.logq_workspace_bytes()
+    ws = logq.new_workspace(nbytes=wsb)
+    items = [(codes, cb, N, None) for (codes, cb, ocb, q), (N, _) in zip(layers, shapes)]
+    outs = logq.logq_linear_grouped(items, X, K, y_dtype=torch.bfloat16, workspace=ws)
+    for (codes, cb, ocb, q), (N, _), Y in zip(layers, shapes, outs):
+        assert torch.equal(Y, logq.logq_linear(codes, cb, X, N, K, y_dtype=torch.bfloat16, workspace=ws))
+        Yr, A = reference(X, q, ocb)
+        check_linear(Y.double().cpu().numpy(), Yr, A, "bf16")
+    st, detail = logq.logq_workspace_status(ws)
+    assert st == logq.LOGQ_OK and detail == 0
+
+
 @pytest.mark.parametrize("ydt", [torch.bfloat16, None])
 def test_prefill_output_dtypes_and_fp16(logq, ydt):
     run_case(logq, 512, 1024, 4, 256, torch.bfloat16, ydt=ydt, seed=5)
