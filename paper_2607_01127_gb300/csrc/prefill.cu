@@ -65,9 +65,9 @@ constexpr int kWStages = 8;              // dequantised weight tiles in flight (
 #define LOGQ_PREFILL_DECODE_WARPS 8
 #endif
 constexpr int kDecodeWarps = LOGQ_PREFILL_DECODE_WARPS;
-static_assert(kDecodeWarps == 8 || kDecodeWarps == 16, "two or four k slices per stage");
+static_assert(kDecodeWarps == 4 || kDecodeWarps == 8 || kDecodeWarps == 16, "one, two or four k slices per stage");
 constexpr int kSlices = kDecodeWarps / 4;
-constexpr int kSliceK = 64 / kSlices;            // k per decode thread and stage: 32 or 16
+constexpr int kSliceK = 64 / kSlices;            // k per decode thread and stage: 64, 32 or 16
 constexpr int kSlicePairs = kSliceK / 2;         // TMEM columns (16-bit pairs) per thread and stage
 constexpr int kDecodeThreads = 32 * kDecodeWarps;
 constexpr int kEpiWarps = 8;                       // two per TMEM lane quarter
@@ -259,6 +259,19 @@ __device__ __forceinline__ void mma_f16_ta(uint32_t tmem_d, uint32_t tmem_a, uin
         : "memory");
 }
 
+[[maybe_unused]] __device__ __forceinline__ void tmem_st_pairs(uint32_t taddr, const uint32_t (&v)[32])
+{
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+        "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+        "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};"
+        ::"r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
+          "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]),
+          "r"(v[16]), "r"(v[17]), "r"(v[18]), "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]),
+          "r"(v[24]), "r"(v[25]), "r"(v[26]), "r"(v[27]), "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31])
+        : "memory");
+}
+
 [[maybe_unused]] __device__ __forceinline__ void tmem_st_pairs(uint32_t taddr, const uint32_t (&v)[8])
 {
     asm volatile(
@@ -331,7 +344,9 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
     static_assert(BN >= 16 && BN <= kBNMax && BN % 16 == 0, "MMA N with M = 128");
     constexpr int XB = BN * kBK * 2;                     // bytes of one X stage
     constexpr int kChunks = ((BN < 128 ? BN : 128) + 31) / 32;   // 32-column drains per epilogue warp
-    constexpr int SLOTS = (EIGHT && kSliceK == 32) ? 2 : 1;   // 16-byte ring slots per thread and stage
+    // 16-byte ring slots per thread and stage: 8-bit kSliceK bytes; 4-bit kSliceK / 2
+    // bytes; 3-bit one 12-byte group per slot (a 16-k slice copies its whole group)
+    constexpr int SLOTS = EIGHT ? (kSliceK >= 16 ? kSliceK / 16 : 1) : (kSliceK == 64 ? 2 : 1);
     // code stages in flight per decode thread: as many as the free halves of the
     // table rows hold, at most 7
     constexpr int RING_FIT = (256 * 128) / (SLOTS * kCodeStageBytes);
@@ -667,15 +682,21 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
                 const uint8_t* src = ahead.row + (int64_t)ahead.ks * step_bytes;
                 const uint32_t dst = ring_slot(g % RING, SLOTS * d);
                 if constexpr (EIGHT) {
-                    cp_async_16(dst, src);
-                    if constexpr (kSliceK == 32) cp_async_16(dst + 16, src + 16);
+#pragma unroll
+                    for (int q = 0; q < SLOTS; ++q) cp_async_16(dst + 16 * q, src + 16 * q);
                 } else if (p.bits == 4) {
-                    if constexpr (kSliceK == 32) cp_async_16(dst, src);
-                    else cp_async_8(dst, src);
+                    if constexpr (kSliceK == 16) cp_async_8(dst, src);
+                    else {
+#pragma unroll
+                        for (int q = 0; q < SLOTS; ++q) cp_async_16(dst + 16 * q, src + 16 * q);
+                    }
                 } else {
-                    cp_async_4(dst, src);
-                    cp_async_4(dst + 4, src + 4);
-                    cp_async_4(dst + 8, src + 8);
+#pragma unroll
+                    for (int q = 0; q < SLOTS; ++q) {                // group q: 12 bytes into slot q
+                        cp_async_4(dst + 16 * q, src + 12 * q);
+                        cp_async_4(dst + 16 * q + 4, src + 12 * q + 4);
+                        cp_async_4(dst + 16 * q + 8, src + 12 * q + 8);
+                    }
                 }
             }
             if (g < total) step(ahead);
@@ -686,14 +707,12 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
             if constexpr (EIGHT) {
                 // word i holds the codes of k = kSliceK h + 4i .. +3: pairs 2i and 2i + 1
                 constexpr int NWD = kSliceK / 4;
-                uint32_t cw8[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-                if (valid) {
-                    const uint4 c0 = lds128(ring_slot(slot, SLOTS * d));
-                    cw8[0] = c0.x; cw8[1] = c0.y; cw8[2] = c0.z; cw8[3] = c0.w;
-                    if constexpr (NWD == 8) {
-                        const uint4 c1 = lds128(ring_slot(slot, SLOTS * d) + 16);
-                        cw8[4] = c1.x; cw8[5] = c1.y; cw8[6] = c1.z; cw8[7] = c1.w;
-                    }
+                uint32_t cw8[NWD];
+#pragma unroll
+                for (int q = 0; q < NWD / 4; ++q) {
+                    uint4 c0 = make_uint4(0, 0, 0, 0);
+                    if (valid) c0 = lds128(ring_slot(slot, SLOTS * d) + 16 * q);
+                    cw8[4 * q] = c0.x; cw8[4 * q + 1] = c0.y; cw8[4 * q + 2] = c0.z; cw8[4 * q + 3] = c0.w;
                 }
 #pragma unroll
                 for (int i = 0; i < NWD; ++i) {
@@ -706,9 +725,13 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
                 }
                 return;
             }
-            uint4 cv = make_uint4(0, 0, 0, 0);
-            if (valid) cv = lds128(ring_slot(slot, d));
-            const uint32_t cw[4] = {cv.x, cv.y, cv.z, cv.w};
+            uint32_t cw[4 * SLOTS];
+#pragma unroll
+            for (int q = 0; q < SLOTS; ++q) {
+                uint4 cv = make_uint4(0, 0, 0, 0);
+                if (valid) cv = lds128(ring_slot(slot, SLOTS * d) + 16 * q);
+                cw[4 * q] = cv.x; cw[4 * q + 1] = cv.y; cw[4 * q + 2] = cv.z; cw[4 * q + 3] = cv.w;
+            }
             if (p.bits == 4) {
                 // word i holds k = kSliceK h + 8i .. +7
 #pragma unroll
@@ -722,16 +745,21 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
             } else {
                 // one 12-byte group of 32 k: pair q (k 2q, 2q + 1) is the 6-bit field q % 5
                 // of word q / 5 (q < 15); pair 15 takes the two top bits of each word
-                auto pair_off = [&](int q) -> uint32_t {
+                // group gi's words are cw[4 gi .. 4 gi + 2] (its ring slot)
+                auto pair_off = [&](int q, int gi = 0) -> uint32_t {
+                    const uint32_t* g3 = cw + 4 * gi;
                     if (q == 15)
-                        return ((cw[0] >> 22) & 0x0300u) | ((cw[1] >> 20) & 0x0c00u) | ((cw[2] >> 18) & 0x3000u) | lane4;
+                        return ((g3[0] >> 22) & 0x0300u) | ((g3[1] >> 20) & 0x0c00u) | ((g3[2] >> 18) & 0x3000u) | lane4;
                     const int f = q % 5;
-                    const uint32_t x = cw[q / 5];
+                    const uint32_t x = g3[q / 5];
                     const uint32_t field = f == 0 ? (x << 8) : f == 1 ? (x << 2) : f == 2 ? (x >> 4)
                                          : f == 3 ? (x >> 10) : (x >> 16);
                     return (field & 0x3f00u) | lane4;
                 };
-                if constexpr (kSliceK == 32) {
+                if constexpr (kSliceK == 64) {
+#pragma unroll
+                    for (int q = 0; q < 32; ++q) pr[q] = lds_tab(pair_off(q & 15, q >> 4));
+                } else if constexpr (kSliceK == 32) {
 #pragma unroll
                     for (int q = 0; q < 16; ++q) pr[q] = lds_tab(pair_off(q));
                 } else {
