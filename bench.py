@@ -783,7 +783,7 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
-CASES = ("decode_layers_8b", "skinny_gate_8b", "gemv_gateup_1b", "gemv_gate_8b", "prefill_q_8b", "quantize_gate_8b", "energy_gate_8b",
+CASES = ("decode_layers_8b", "decode_step_1b", "skinny_gate_8b", "gemv_gateup_1b", "gemv_gate_8b", "prefill_q_8b", "quantize_gate_8b", "energy_gate_8b",
          "gemv8_gate_8b", "gptq_q_8b", "gptq_update_q_8b", "quantize3_gate_8b")
 
 
@@ -802,6 +802,13 @@ def run_case(name: str):
         # the first two layers of the 8B decode step (8 chained launches, each
         # warming L2 with the next one's codes), run twice
         launches, ws, arena, _ = build_decode_model(logq, torch, dev, layers=2)
+        stream = torch.cuda.Stream(device=dev)
+        for _ in range(2):
+            step_graph(logq, torch, launches, ws, stream)
+        torch.cuda.synchronize()
+    elif name == "decode_step_1b":
+        # the Llama-3.2-1B decode step (64 chained launches), run twice
+        launches, ws, arena, _ = build_decode_model(logq, torch, dev, "1b")
         stream = torch.cuda.Stream(device=dev)
         for _ in range(2):
             step_graph(logq, torch, launches, ws, stream)
