@@ -184,7 +184,44 @@ def cpu_baseline(seconds: float = 12.0):
     dt = time.perf_counter() - t0
     return {"value": round(nbytes / dt / 1e9, 4), "unit": "GB/s", "cores": threads, "kind": "oracle",
             "sample": f"fp64 oracle GEMV over the first 8 rows of all {len(items)} linears of the decode "
-                      f"step, {reps} passes in {dt:.1f} s"}
+                      f"step, {reps} passes in {dt:.1f} s",
+            "rates": oracle_rates(threads)}
+
+
+def oracle_rates(threads: int, seconds: float = 1.5):
+    """The oracle's other rates on the host cores, one core and all of them: the
+    GEMV sample in GB/s, quantisation (Eq. (1) through fp64 logarithms) in
+    weights/s, and the fp64 product of a 2048-token prefill slice in GFLOP/s."""
+    import oracle
+    from concurrent.futures import ThreadPoolExecutor
+
+    def rate(fn, units):
+        fn()
+        t0, n = time.perf_counter(), 0
+        while time.perf_counter() - t0 < seconds:
+            fn()
+            n += 1
+        return units * n / (time.perf_counter() - t0)
+
+    out = {"cores_all": threads}
+    items = oracle_gemv_sample()
+    gb = oracle_gemv_run(items, 1)
+    out["gemv_gbs_1core"] = round(rate(lambda: oracle_gemv_run(items, 1), gb) / 1e9, 4)
+    w = workloads.weights_np(512, 4096, 21, outliers=True)
+    cb = oracle.build_codebook(4, 1.5, float(np.abs(w).max()))
+    out["quantize_weights_per_s_1core"] = round(rate(lambda: oracle.quantize_log(w, cb), w.size), 1)
+    chunks = np.array_split(w, threads)                 # the C call releases the GIL
+    with ThreadPoolExecutor(threads) as ex:
+        out["quantize_weights_per_s_all"] = round(
+            rate(lambda: list(ex.map(lambda c: oracle.quantize_log(c, cb), chunks)), w.size), 1)
+    X = workloads.activations_np(16, 4096, 22).astype(np.float64)
+    What = oracle.dequant(oracle.quantize_log(w, cb), cb)
+    fl = 2.0 * X.shape[0] * What.shape[0] * X.shape[1]
+    out["prefill_gflops_1core"] = round(rate(lambda: oracle.linear(X, What, 1), fl) / 1e9, 3)
+    out["prefill_gflops_all"] = round(rate(lambda: oracle.linear(X, What, threads), fl) / 1e9, 3)
+    out["note"] = ("GEMV: the sample above; quantise: 512 x 4096 Student-t weights, 4-bit; prefill: 16 "
+                   "tokens x 512 x 4096 of a 2048-token batch (fp64, the oracle's own loops)")
+    return out
 
 
 def run_reference(args):
@@ -611,17 +648,21 @@ def run_ours(args):
     for _ in range(args.warmup):
         graph.replay()
     barrier()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    # one event before the first replay and one after each: the whole region's
+    # time (the value) and each step's (median and best)
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    e0, e1 = evs[0], evs[-1]
     with ClockSampler(local) as clocks:
         time.sleep(0.25)
         barrier()
         with torch.cuda.stream(stream):
             e0.record(stream)
-            for _ in range(args.steps):
+            for i in range(args.steps):
                 graph.replay()
-            e1.record(stream)
+                evs[i + 1].record(stream)
         barrier()
         time.sleep(0.25)
+    per_step = sorted(evs[i].elapsed_time(evs[i + 1]) for i in range(args.steps))
     t, total_bytes = replica_totals(e0.elapsed_time(e1) * 1e-3, step_bytes * args.steps, dist, dev)
     value = total_bytes / t / 1e9
     ms_per_step = t / args.steps * 1e3
@@ -671,6 +712,8 @@ def run_ours(args):
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": "GB/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4),
+        "step_ms": {"median": round(per_step[len(per_step) // 2], 4), "best": round(per_step[0], 4),
+                    "worst": round(per_step[-1], 4), "note": "this rank's steps, one event pair each"},
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic",
         "config": {"workload": WORKLOAD, "global_batch": 1 * world, "linears_per_step": n_linears,
@@ -681,7 +724,8 @@ def run_ours(args):
                    "graph": "one CUDA graph per step: per layer qkv | o | gate+up | down launches "
                             "(linears that read the same activations share a launch), chained: each "
                             "launch reads the previous launch's bf16 output; programmatic dependent "
-                            "launch, each launch warms L2 with the next launch's codes"},
+                            "launch, each launch warms L2 with the next launch's codes when they are "
+                            "under 20 MiB"},
         "e2e": {"value": round(e2e_value, 1), "unit": "GB/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": launches_per_step * args.steps,
