@@ -444,6 +444,36 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         return e < ksteps ? e : ksteps;
     };
 
+    // the code rows of a tile are one contiguous block: ask L2 for it one
+    // tile ahead so the decode warps' copies hit L2.  An epilogue warp issues
+    // it: from the producer warp it delays the X loads behind it, and a CTA's
+    // first tile is not prefetched, since its copies would only compete with
+    // the decode warps' own loads of the same rows.
+    auto prefetch_codes = [&](int tile) {
+        if (tile >= ntiles) return;
+        const int64_t n0 = (int64_t)tile_n(tile) * kBM;
+        const int64_t rows = (p.N - n0) < kBM ? (p.N - n0) : kBM;
+        const uint8_t* base = p.codes + n0 * p.row_bytes;
+        if (p.splits == 1) {
+            const int64_t bytes = rows * p.row_bytes;
+            for (int64_t off = (int64_t)lane * 16384; off < bytes; off += 32 * 16384) {
+                const int64_t nb = (bytes - off) < 16384 ? (bytes - off) : 16384;
+                asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base + off), "r"((uint32_t)nb)
+                             : "memory");
+            }
+            return;
+        }
+        // the tile's k range of each row, widened to 16-byte bounds inside the row
+        // (row_bytes is a multiple of 16, and of the k-step count)
+        const int64_t step_bytes = p.row_bytes / ksteps;
+        const int64_t b0 = ((int64_t)k_begin(tile) * step_bytes) & ~(int64_t)15;
+        int64_t b1 = ((int64_t)k_end(tile) * step_bytes + 15) & ~(int64_t)15;
+        if (b1 > p.row_bytes) b1 = p.row_bytes;
+        for (int64_t r = lane; r < rows; r += 32)
+            asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base + r * p.row_bytes + b0),
+                         "r"((uint32_t)(b1 - b0))
+                         : "memory");
+    };
     if (warp == 0) {
         // ---------------- TMA producer ----------------
         // The whole warp walks the loop (uniform operands); one elected lane issues.
@@ -451,37 +481,8 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         uint32_t phase = 0;
         bool ok = true;
         uint32_t issued = 0, issued_par = 0;           // per stage: used at least once / parity of last load
-        // the code rows of a tile are one contiguous block: ask L2 for it one
-        // tile ahead so the decode warps' copies hit L2
-        auto prefetch_codes = [&](int tile) {
-            if (tile >= ntiles) return;
-            const int64_t n0 = (int64_t)tile_n(tile) * kBM;
-            const int64_t rows = (p.N - n0) < kBM ? (p.N - n0) : kBM;
-            const uint8_t* base = p.codes + n0 * p.row_bytes;
-            if (p.splits == 1) {
-                const int64_t bytes = rows * p.row_bytes;
-                for (int64_t off = (int64_t)lane * 16384; off < bytes; off += 32 * 16384) {
-                    const int64_t nb = (bytes - off) < 16384 ? (bytes - off) : 16384;
-                    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base + off), "r"((uint32_t)nb)
-                                 : "memory");
-                }
-                return;
-            }
-            // the tile's k range of each row, widened to 16-byte bounds inside the row
-            // (row_bytes is a multiple of 16, and of the k-step count)
-            const int64_t step_bytes = p.row_bytes / ksteps;
-            const int64_t b0 = ((int64_t)k_begin(tile) * step_bytes) & ~(int64_t)15;
-            int64_t b1 = ((int64_t)k_end(tile) * step_bytes + 15) & ~(int64_t)15;
-            if (b1 > p.row_bytes) b1 = p.row_bytes;
-            for (int64_t r = lane; r < rows; r += 32)
-                asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base + r * p.row_bytes + b0),
-                             "r"((uint32_t)(b1 - b0))
-                             : "memory");
-        };
-        prefetch_codes(blockIdx.x);
         for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
             const int t0 = tile_t(tile) * BN;
-            prefetch_codes(tile + gridDim.x);
             const int kb = k_begin(tile), ke = k_end(tile);
             for (int ks = kb; ks < ke; ++ks) {
                 if (!warp_wait(xempty(stage), phase ^ 1u, abort_flag, p.ws, kWaitProducer)) {
@@ -564,7 +565,10 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         const int row = quarter * 32 + lane;
         const uint32_t tq = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(ehalf * 128);
         int it = 0;
+        // an epilogue warp of the second column half, idle in 16-token tiles
+        const bool pf_warp = warp == kEpi0 + 4;
         for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
+            if (pf_warp) prefetch_codes(tile + gridDim.x);
             if (!warp_wait(accfull, (uint32_t)it & 1u, abort_flag, p.ws, kWaitEpilogue)) break;
             tc_fence_after();
             const int64_t n = (int64_t)tile_n(tile) * kBM + row;
