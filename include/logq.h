@@ -321,7 +321,14 @@ typedef struct logq_linear_item {
  * with its own per-tensor codebook (Sec. 3.1) and output: Y_i = X * What_i^T
  * (Sec. 3.3), in one call.  count is 1..4 and all items share the code width
  * of their codebooks.  With B <= 16 (4-bit) or B <= 4 (3-, 8-bit) the matrices
- * share a single decode-GEMV launch; larger B runs one prefill launch each.
+ * share a single decode-GEMV launch.  Larger B (and 4-bit batches of 8..16
+ * that logq_linear would send to the tensor cores) runs one prefill launch
+ * whose CTAs are divided among the matrices in proportion to their tiles,
+ * when its estimate beats one launch per matrix (small matrices such as k / v
+ * projections then share the GPU with a larger one); otherwise one launch
+ * each, as logq_linear.  The workspace holds the partial sums of split k
+ * ranges as for logq_linear: logq_linear_grouped_workspace_bytes gives the
+ * size with which the planned launches split fully.
  * l2_prefetch (device, may be NULL) / l2_prefetch_bytes name a range the
  * call asks the L2 cache to fetch while it runs -- for a decode step, the
  * codes of the next layer -- a hint only: it is never read by the
@@ -337,6 +344,13 @@ logq_status logq_linear_grouped(const logq_linear_item* items, int count, const 
                                 logq_dtype x_dtype, int64_t B, int64_t K, logq_dtype y_dtype,
                                 const void* l2_prefetch, size_t l2_prefetch_bytes,
                                 void* workspace, size_t workspace_bytes, void* stream);
+
+/* Workspace bytes with which logq_linear_grouped of count (1..4) matrices of
+ * N[0..count-1] rows (host array), code width bits and batch B runs as
+ * planned: logq_workspace_bytes() plus the largest partial-sum space among
+ * its launches.  A smaller workspace (at least logq_workspace_bytes()) is
+ * accepted and only reduces the splits.  0 for invalid sizes. */
+size_t logq_linear_grouped_workspace_bytes(int64_t B, const int64_t* N, int count, int64_t K, int bits);
 
 /* Synchronise `stream`, read the device error word of `workspace`, clear it,
  * and return LOGQ_OK or LOGQ_ERR_TIMEOUT.  *detail (host, may be NULL)

@@ -38,7 +38,7 @@ LOGQ_F32, LOGQ_BF16, LOGQ_F16 = 0, 1, 2
 LOGQ_SHIFT_EXACT, LOGQ_SHIFT_FLOOR = 0, 1
 
 EXPORTED = ("logq_build_codebook", "logq_packed_bytes", "logq_workspace_bytes", "logq_linear_workspace_bytes",
-            "logq_quantize",
+            "logq_linear_grouped_workspace_bytes", "logq_quantize",
             "logq_linear", "logq_workspace_status", "logq_status_string", "logq_device_sm_count",
             "logq_quantize_noalloc", "logq_linear_grouped", "logq_energy_scratch_bytes",
             "logq_quantize_energy", "logq_gptq_factor_scratch_bytes", "logq_gptq_factor",
@@ -91,6 +91,8 @@ def _load() -> ctypes.CDLL:
     lib.logq_workspace_bytes.restype = ctypes.c_size_t
     lib.logq_linear_workspace_bytes.argtypes = [c_i64, c_i64, c_i64, c_int]
     lib.logq_linear_workspace_bytes.restype = ctypes.c_size_t
+    lib.logq_linear_grouped_workspace_bytes.argtypes = [c_i64, ctypes.POINTER(c_i64), c_int, c_i64, c_int]
+    lib.logq_linear_grouped_workspace_bytes.restype = ctypes.c_size_t
     lib.logq_quantize.argtypes = [P, c_i64, c_i64, c_int, c_dbl, c_dbl, c_int, P,
                                   ctypes.POINTER(Codebook), P, ctypes.c_size_t, P]
     lib.logq_quantize.restype = c_int
@@ -187,6 +189,11 @@ def logq_workspace_bytes() -> int:
 
 def logq_linear_workspace_bytes(B: int, N: int, K: int, bits: int) -> int:
     return int(_lib().logq_linear_workspace_bytes(int(B), int(N), int(K), int(bits)))
+
+
+def logq_linear_grouped_workspace_bytes(B: int, Ns, K: int, bits: int) -> int:
+    arr = (ctypes.c_int64 * len(Ns))(*[int(n) for n in Ns])
+    return int(_lib().logq_linear_grouped_workspace_bytes(int(B), arr, len(Ns), int(K), int(bits)))
 
 
 def new_workspace(device=None, nbytes: int | None = None):
@@ -330,7 +337,7 @@ def logq_linear(codes, cb: Codebook, X, N: int, K: int, y_dtype=None, Y=None, wo
 
 def logq_linear_grouped(items, X, K: int, y_dtype=None, workspace=None, prefetch=None,
                         prefetch_bytes: int = 0, stream=None):
-    """One launch for up to four matrices sharing X: items = [(codes, cb, N, Y or None), ...].
+    """Up to four matrices sharing X in one launch: items = [(codes, cb, N, Y or None), ...].
     prefetch: optional device tensor (or (tensor, bytes)) the call warms L2 with.
     Returns the list of outputs."""
     import torch
@@ -351,8 +358,8 @@ def logq_linear_grouped(items, X, K: int, y_dtype=None, workspace=None, prefetch
         arr[i] = LinearItem(ctypes.c_void_p(codes.data_ptr()), ctypes.pointer(cb), int(N),
                             ctypes.c_void_p(Y.data_ptr()))
     if workspace is None:
-        workspace = new_workspace(X.device, max(logq_linear_workspace_bytes(B, int(N), K, cb.bits)
-                                                for _, cb, N, _ in items))
+        workspace = new_workspace(X.device, logq_linear_grouped_workspace_bytes(
+            B, [int(N) for _, _, N, _ in items], K, items[0][1].bits))
     pf_ptr = ctypes.c_void_p(prefetch.data_ptr()) if prefetch is not None else None
     pf_bytes = int(prefetch_bytes) if prefetch is not None else 0
     st = _lib().logq_linear_grouped(arr, len(items), ctypes.c_void_p(X.data_ptr()), xd, B, int(K), yd, pf_ptr,

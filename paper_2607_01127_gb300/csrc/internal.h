@@ -115,16 +115,22 @@ cudaError_t launch_gptq_factor(const float* H, int64_t K, double damp, float* U,
                                uint32_t* not_pd, cudaStream_t s);
 cudaError_t launch_gemv_group(const GroupArgs& a, cudaStream_t s);
 cudaError_t launch_prefill(const LinearArgs& a, cudaStream_t s);
-// Tensor-core launch plan of a B x N x K product: token-tile width, k ranges per
-// output tile (the partial sums need part_bytes of workspace beyond
-// kWorkspaceBytes; at most part_bytes_avail are used).
+// One tensor-core launch over the group's matrices (ws_bytes: the caller's
+// workspace, which holds the split k ranges' partial sums).
+cudaError_t launch_prefill_group(const GroupArgs& g, size_t ws_bytes, cudaStream_t s);
+// Tensor-core launch plan of B x N[i] x K products sharing X (count <= 4):
+// token-tile width, k ranges per output tile (the partial sums need part_bytes
+// of workspace beyond kWorkspaceBytes; at most part_bytes_avail are used) and
+// the CTAs each matrix gets.
 struct PrefillPlan {
     int bn;
     int splits;
     int ksplit;
     size_t part_bytes;
     double est_us;          // estimated launch time on a GB300 (planning only)
+    int ncta[4];
 };
+PrefillPlan prefill_plan(int64_t B, const int64_t* N, int count, int64_t K, size_t part_bytes_avail);
 PrefillPlan prefill_plan(int64_t B, int64_t N, int64_t K, size_t part_bytes_avail);
 bool gemv_supports(int bits, int64_t B);
 

@@ -155,13 +155,63 @@ bool tensor_core_batch(int bits, int64_t B)
 // FMAs bound it), plus ~2 us per launch (measured on the GB300 on the
 // Llama-3.1-8B shapes).  The tensor-core estimate depends on how far the caller's
 // workspace lets the k ranges split (prefill_plan).
+double cuda_core_us(int64_t B, int64_t N, int64_t K)
+{
+    return (double)N * (double)K * (B <= 8 ? 0.46e-6 : 0.84e-6) + 2.0;
+}
+
 bool use_small_batch_tc(int bits, int64_t B, int64_t N, int64_t K, size_t workspace_bytes)
 {
     if (!(bits == 4 && B >= LOGQ_TC_MIN_BATCH && B <= 16)) return false;
     const size_t avail = workspace_bytes > kWorkspaceBytes ? workspace_bytes - kWorkspaceBytes : 0;
     const PrefillPlan pl = prefill_plan(B, N, K, avail);
-    const double cuda_us = (double)N * (double)K * (B <= 8 ? 0.46e-6 : 0.84e-6) + 2.0;
-    return pl.est_us < cuda_us;
+    return pl.est_us < cuda_core_us(B, N, K);
+}
+
+// How a grouped call runs: one CUDA-core launch over all matrices, one
+// tensor-core launch whose CTAs the matrices share (small ones, such as k / v
+// projections, then no longer leave SMs idle), or each matrix as its own
+// logq_linear call -- whichever is estimated fastest; batches the CUDA-core
+// kernel always takes stay there.  A smaller workspace can only slow the
+// options that split k ranges, so the workspace the choice needs
+// (part_bytes) leads to the same choice.
+struct GroupChoice {
+    enum { kCudaCores, kTensorCores, kSingles } kind;
+    size_t part_bytes;
+};
+
+GroupChoice choose_group(int bits, int64_t B, const int64_t* N, int count, int64_t K, size_t workspace_bytes)
+{
+    GroupChoice ch{GroupChoice::kCudaCores, 0};
+    if (!tensor_core_batch(bits, B)) return ch;
+    const size_t avail = workspace_bytes > kWorkspaceBytes ? workspace_bytes - kWorkspaceBytes : 0;
+    const bool cuda_ok = gemv_supports(bits, B);
+    double cuda_us = 2.0, singles_us = 0.0;
+    size_t single_part = 0;
+    for (int i = 0; i < count; ++i) {
+        const PrefillPlan pl = prefill_plan(B, N[i], K, avail);
+        double us = pl.est_us;
+        size_t part = pl.part_bytes;
+        if (cuda_ok) {
+            const double c = cuda_core_us(B, N[i], K);
+            cuda_us += c - 2.0;
+            if (c <= us) {
+                us = c;
+                part = 0;
+            }
+        }
+        singles_us += us;
+        single_part = part > single_part ? part : single_part;
+    }
+    const PrefillPlan gp = prefill_plan(B, N, count, K, avail);
+    double best = cuda_ok ? cuda_us : 1e300;
+    if (count > 1 && gp.est_us < best) {
+        best = gp.est_us;
+        ch = GroupChoice{GroupChoice::kTensorCores, gp.part_bytes};
+    }
+    if (singles_us < best)
+        ch = GroupChoice{GroupChoice::kSingles, single_part};
+    return ch;
 }
 
 }  // namespace
@@ -237,6 +287,14 @@ size_t logq_linear_workspace_bytes(int64_t B, int64_t N, int64_t K, int bits)
     if (!tensor_core_batch(bits, B)) return kWorkspaceBytes;
     if (gemv_supports(bits, B) && !use_small_batch_tc(bits, B, N, K, (size_t)-1)) return kWorkspaceBytes;
     return kWorkspaceBytes + prefill_plan(B, N, K, (size_t)-1).part_bytes;
+}
+
+size_t logq_linear_grouped_workspace_bytes(int64_t B, const int64_t* N, int count, int64_t K, int bits)
+{
+    if (!N || count < 1 || count > 4 || B <= 0) return 0;
+    for (int i = 0; i < count; ++i)
+        if (logq_packed_bytes(N[i], K, bits) == 0) return 0;
+    return kWorkspaceBytes + choose_group(bits, B, N, count, K, (size_t)-1).part_bytes;
 }
 
 logq_status logq_quantize(const float* W, int64_t N, int64_t K, int bits, double base,
@@ -408,28 +466,34 @@ logq_status logq_linear_grouped(const logq_linear_item* items, int count, const 
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     Workspace* ws = static_cast<Workspace*>(workspace);
     const int x_f16 = (x_dtype == LOGQ_F16);
-    bool all_tc = true;                     // every item takes the small-batch tensor-core path
-    for (int i = 0; i < count; ++i) all_tc = all_tc && use_small_batch_tc(bits, B, items[i].N, K, workspace_bytes);
-    if (gemv_supports(bits, B) && !all_tc) {
-        GroupArgs g;
-        memset(&g, 0, sizeof g);
-        g.count = count;
-        for (int i = 0; i < count; ++i) {
-            g.item[i].codes = items[i].codes;
-            g.item[i].Y = items[i].Y;
-            g.item[i].N = items[i].N;
-            const uint16_t* tab = x_f16 ? items[i].cb->level_f16 : items[i].cb->level_bf16;
-            for (int c = 0; c < (1 << bits); ++c) g.item[i].lvl16[c] = tab[c];
-        }
-        g.X = X;
-        g.B = B;
-        g.K = K;
-        g.bits = bits;
-        g.x_f16 = x_f16;
-        g.y_dtype = (int)y_dtype;
+    GroupArgs g;
+    memset(&g, 0, sizeof g);
+    g.count = count;
+    for (int i = 0; i < count; ++i) {
+        g.item[i].codes = items[i].codes;
+        g.item[i].Y = items[i].Y;
+        g.item[i].N = items[i].N;
+        const uint16_t* tab = x_f16 ? items[i].cb->level_f16 : items[i].cb->level_bf16;
+        for (int c = 0; c < (1 << bits); ++c) g.item[i].lvl16[c] = tab[c];
+    }
+    g.X = X;
+    g.B = B;
+    g.K = K;
+    g.bits = bits;
+    g.x_f16 = x_f16;
+    g.y_dtype = (int)y_dtype;
+    g.ws = ws;
+    int64_t Ns[4];
+    for (int i = 0; i < count; ++i) Ns[i] = items[i].N;
+    const GroupChoice ch = choose_group(bits, B, Ns, count, K, workspace_bytes);
+    if (ch.kind == GroupChoice::kCudaCores) {
         aligned_prefetch_range(l2_prefetch, l2_prefetch_bytes, &g.pf, &g.pf_bytes);
-        g.ws = ws;
         return cuda_status(launch_gemv_group(g, s));
+    }
+    if (ch.kind == GroupChoice::kTensorCores) {
+        const cudaError_t e = launch_prefill_group(g, workspace_bytes, s);
+        if (e == cudaErrorNotSupported) return LOGQ_ERR_UNSUPPORTED;
+        return cuda_status(e);
     }
     for (int i = 0; i < count; ++i) {
         const logq_status st = logq_linear(items[i].codes, items[i].cb, X, x_dtype, B, items[i].N, K, items[i].Y,

@@ -54,6 +54,7 @@ namespace {
 constexpr int kBM = 128;                 // weight rows per tile (MMA M)
 constexpr int kBNMax = 256;              // widest token tile (MMA N)
 constexpr int kBK = 64;                  // k per stage (one 128-byte swizzle atom of bf16)
+constexpr int kMaxPrefillItems = 4;      // matrices of one grouped launch
 constexpr int kXStages = 5;              // X tiles in flight (TMA)
 constexpr int kWStages = 8;              // dequantised weight tiles in flight (tensor memory)
 // Decode warps: four per k slice of a stage (one per TMEM lane quarter), each
@@ -93,22 +94,34 @@ enum : uint32_t { kWaitProducer = 1, kWaitMma = 2, kWaitEpilogue = 3, kWaitDecod
 constexpr uint32_t kTestStallWord = 0x57A11u;   // workspace reserved[0] value that triggers the test stall
 #endif
 
-struct PrefillParams {
+// One matrix of a launch.  A grouped launch (matrices sharing X) gives each
+// matrix a contiguous range of CTAs, in proportion to its tiles; a CTA works
+// on its matrix's tiles only, so it builds one pair table.
+struct PrefillItem {
     const uint8_t* codes;
     void* Y;
-    Workspace* ws;
     float* part;            // splits > 1: fp32 partial sums [splits][B][N] (caller's workspace)
     int64_t N;
+    int32_t n_tiles_n;
+    int32_t cta_begin;      // first CTA of this matrix
+    int32_t ncta;           // its CTAs
+    int32_t pad_;
+    uint16_t lvl16[256];    // code-indexed 16-bit levels (2^bits used)
+};
+
+struct PrefillParams {
+    PrefillItem item[kMaxPrefillItems];
+    int32_t nitems;
+    Workspace* ws;
     int32_t K, B;
     int64_t row_bytes;
     int32_t bits;
     int32_t y_dtype;
-    int32_t n_tiles_n, n_tiles_t;
-    int32_t splits;         // k ranges per output tile
+    int32_t n_tiles_t;
+    int32_t splits;         // k ranges per output tile (the same for every matrix)
     int32_t ksplit;         // k-steps per range (the last may be shorter)
     uint32_t idesc;
     uint32_t smem_bytes;    // dynamic shared memory of the launch (layout check)
-    uint16_t lvl16[256];    // code-indexed 16-bit levels (2^bits used)
 };
 
 // ------------------------------------------------------------------ PTX ---
@@ -389,6 +402,16 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
     volatile int* abort_flag = reinterpret_cast<volatile int*>(gen + tmem_slot + 8);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    // this CTA's matrix, and its place among that matrix's CTAs
+    int m = 0;
+#pragma unroll
+    for (int i = 1; i < kMaxPrefillItems; ++i)
+        if (i < p.nitems && (int)blockIdx.x >= p.item[i].cta_begin) m = i;
+    const PrefillItem& item = p.item[m];
+    const int cta = (int)blockIdx.x - item.cta_begin, ncta = item.ncta;
+    const uint8_t* const codes = item.codes;
+    const int64_t N = item.N;
+    const int n_tiles_n = item.n_tiles_n;
     if (tid == 0) {
         for (int s = 0; s < kXStages; ++s) {
             mbar_init(xfull(s), 1);
@@ -412,11 +435,11 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
             const int e = i >> 3, part = i & 7;
             uint32_t v;
             if constexpr (EIGHT) {
-                v = (uint32_t)p.lvl16[e] * 0x10001u;
+                v = (uint32_t)item.lvl16[e] * 0x10001u;
             } else {
                 const uint32_t lo = (p.bits == 4) ? (e & 15) : (e & 7);
                 const uint32_t hi = (p.bits == 4) ? (e >> 4) : (e >> 3);
-                v = (uint32_t)p.lvl16[lo] | ((uint32_t)p.lvl16[hi] << 16);
+                v = (uint32_t)item.lvl16[lo] | ((uint32_t)item.lvl16[hi] << 16);
             }
             sts128(sbase + e * kTabRow + part * 16, v, v, v, v);
         }
@@ -433,11 +456,11 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
     const uint32_t tmem_base = *reinterpret_cast<volatile uint32_t*>(gen + tmem_slot);
 
     const int ksteps = p.K / kBK;
-    const int ntiles = p.n_tiles_n * p.n_tiles_t * p.splits;
+    const int ntiles = n_tiles_n * p.n_tiles_t * p.splits;
     // tile -> (weight-row tile, token tile, k range); the weight-row tile varies fastest
-    auto tile_n = [&](int tile) { return tile % p.n_tiles_n; };
-    auto tile_t = [&](int tile) { return (tile / p.n_tiles_n) % p.n_tiles_t; };
-    auto tile_sp = [&](int tile) { return tile / (p.n_tiles_n * p.n_tiles_t); };
+    auto tile_n = [&](int tile) { return tile % n_tiles_n; };
+    auto tile_t = [&](int tile) { return (tile / n_tiles_n) % p.n_tiles_t; };
+    auto tile_sp = [&](int tile) { return tile / (n_tiles_n * p.n_tiles_t); };
     auto k_begin = [&](int tile) { return tile_sp(tile) * p.ksplit; };
     auto k_end = [&](int tile) {
         const int e = (tile_sp(tile) + 1) * p.ksplit;
@@ -452,8 +475,8 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
     auto prefetch_codes = [&](int tile) {
         if (tile >= ntiles) return;
         const int64_t n0 = (int64_t)tile_n(tile) * kBM;
-        const int64_t rows = (p.N - n0) < kBM ? (p.N - n0) : kBM;
-        const uint8_t* base = p.codes + n0 * p.row_bytes;
+        const int64_t rows = (N - n0) < kBM ? (N - n0) : kBM;
+        const uint8_t* base = codes + n0 * p.row_bytes;
         if (p.splits == 1) {
             const int64_t bytes = rows * p.row_bytes;
             for (int64_t off = (int64_t)lane * 16384; off < bytes; off += 32 * 16384) {
@@ -481,7 +504,7 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         uint32_t phase = 0;
         bool ok = true;
         uint32_t issued = 0, issued_par = 0;           // per stage: used at least once / parity of last load
-        for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+        for (int tile = cta; tile < ntiles && ok; tile += ncta) {
             const int t0 = tile_t(tile) * BN;
             const int kb = k_begin(tile), ke = k_end(tile);
             for (int ks = kb; ks < ke; ++ks) {
@@ -521,7 +544,7 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         if (p.ws->reserved[0] == kTestStallWord)
             ok = warp_wait(drainb, 0, abort_flag, p.ws, kWaitMma);
 #endif
-        for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
+        for (int tile = cta; tile < ntiles && ok; tile += ncta, ++it) {
             // one accumulator: the epilogue has read the previous tile's out of it
             if (!warp_wait(accempty, ((uint32_t)it & 1u) ^ 1u, abort_flag, p.ws, kWaitMma)) break;
             tc_fence_after();
@@ -567,8 +590,8 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         int it = 0;
         // an epilogue warp of the second column half, idle in 16-token tiles
         const bool pf_warp = warp == kEpi0 + 4;
-        for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
-            if (pf_warp) prefetch_codes(tile + gridDim.x);
+        for (int tile = cta; tile < ntiles; tile += ncta, ++it) {
+            if (pf_warp) prefetch_codes(tile + ncta);
             if (!warp_wait(accfull, (uint32_t)it & 1u, abort_flag, p.ws, kWaitEpilogue)) break;
             tc_fence_after();
             const int64_t n = (int64_t)tile_n(tile) * kBM + row;
@@ -583,17 +606,17 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
                 if (lane == 0) mbar_arrive(accempty);
             } else if (p.splits > 1 || p.y_dtype == LOGQ_F32) {
                 // fp32 out: Y itself, or this k range's partial sums
-                float* yb = p.splits > 1 ? p.part + (int64_t)tile_sp(tile) * p.B * p.N : static_cast<float*>(p.Y);
+                float* yb = p.splits > 1 ? item.part + (int64_t)tile_sp(tile) * p.B * N : static_cast<float*>(item.Y);
 #pragma unroll 1
                 for (int c = 0; c < kChunks; ++c) {
                     uint32_t v[32];
                     tmem_ld32(tq + (uint32_t)(c * 32), v);
                     const int jm = jmax - 32 * c;
-                    if (n < p.N && jm > 0) {
-                        float* y = yb + (int64_t)(tb0 + 32 * c) * p.N + n;
+                    if (n < N && jm > 0) {
+                        float* y = yb + (int64_t)(tb0 + 32 * c) * N + n;
 #pragma unroll
                         for (int j = 0; j < 32; ++j)
-                            if (j < jm) y[(int64_t)j * p.N] = __uint_as_float(v[j]);
+                            if (j < jm) y[(int64_t)j * N] = __uint_as_float(v[j]);
                     }
                 }
                 tc_fence_before();
@@ -621,21 +644,21 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(accempty);
-                if (n < p.N && jmax > 0) {
+                if (n < N && jmax > 0) {
                     // lanes hold consecutive n: each store instruction writes one
                     // contiguous run of Y[t][n0 .. n0+31]
-                    uint16_t* y = static_cast<uint16_t*>(p.Y) + (int64_t)tb0 * p.N + n;
+                    uint16_t* y = static_cast<uint16_t*>(item.Y) + (int64_t)tb0 * N + n;
                     if (jmax == 128) {
 #pragma unroll
                         for (int j = 0; j < 64; ++j) {
-                            y[(int64_t)(2 * j) * p.N] = (uint16_t)(pk[j] & 0xffffu);
-                            y[(int64_t)(2 * j + 1) * p.N] = (uint16_t)(pk[j] >> 16);
+                            y[(int64_t)(2 * j) * N] = (uint16_t)(pk[j] & 0xffffu);
+                            y[(int64_t)(2 * j + 1) * N] = (uint16_t)(pk[j] >> 16);
                         }
                     } else {
 #pragma unroll
                         for (int j = 0; j < 64; ++j) {
-                            if (2 * j < jmax) y[(int64_t)(2 * j) * p.N] = (uint16_t)(pk[j] & 0xffffu);
-                            if (2 * j + 1 < jmax) y[(int64_t)(2 * j + 1) * p.N] = (uint16_t)(pk[j] >> 16);
+                            if (2 * j < jmax) y[(int64_t)(2 * j) * N] = (uint16_t)(pk[j] & 0xffffu);
+                            if (2 * j + 1 < jmax) y[(int64_t)(2 * j + 1) * N] = (uint16_t)(pk[j] >> 16);
                         }
                     }
                 }
@@ -659,7 +682,7 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
         int stage = 0;
         uint32_t phase = 0;
         int total = 0;                                  // stages this CTA decodes
-        for (int t = (int)blockIdx.x; t < ntiles; t += (int)gridDim.x) total += k_end(t) - k_begin(t);
+        for (int t = cta; t < ntiles; t += ncta) total += k_end(t) - k_begin(t);
         // Cursor over (tile, k-step) advanced without divisions: one for the
         // copies issued ahead, one for the stage being decoded.
         struct Cursor {
@@ -672,15 +695,15 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
             c.ks = tile < ntiles ? k_begin(tile) : 0;
             c.ke = tile < ntiles ? k_end(tile) : 0;
             const int64_t n = (int64_t)tile_n(tile) * kBM + r;
-            c.valid = tile < ntiles && n < p.N;
-            c.row = p.codes + (c.valid ? n : 0) * p.row_bytes + slice_off;
+            c.valid = tile < ntiles && n < N;
+            c.row = codes + (c.valid ? n : 0) * p.row_bytes + slice_off;
         };
         auto step = [&](Cursor& c) {
-            if (++c.ks >= c.ke) set_tile(c, c.tile + (int)gridDim.x);
+            if (++c.ks >= c.ke) set_tile(c, c.tile + ncta);
         };
         Cursor ahead, cur;
-        set_tile(ahead, (int)blockIdx.x);
-        set_tile(cur, (int)blockIdx.x);
+        set_tile(ahead, cta);
+        set_tile(cur, cta);
         auto issue = [&](int g) {
             if (g < total && ahead.valid) {
                 const uint8_t* src = ahead.row + (int64_t)ahead.ks * step_bytes;
@@ -727,53 +750,53 @@ prefill_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ 
                     pr[2 * i] = prmt(v0, v1, 0x5410u);
                     pr[2 * i + 1] = prmt(v2, v3, 0x5410u);
                 }
-                return;
-            }
-            uint32_t cw[4 * SLOTS];
-#pragma unroll
-            for (int q = 0; q < SLOTS; ++q) {
-                uint4 cv = make_uint4(0, 0, 0, 0);
-                if (valid) cv = lds128(ring_slot(slot, SLOTS * d) + 16 * q);
-                cw[4 * q] = cv.x; cw[4 * q + 1] = cv.y; cw[4 * q + 2] = cv.z; cw[4 * q + 3] = cv.w;
-            }
-            if (p.bits == 4) {
-                // word i holds k = kSliceK h + 8i .. +7
-#pragma unroll
-                for (int i = 0; i < kSliceK / 8; ++i) {
-                    const uint32_t c = cw[i];
-                    pr[4 * i + 0] = lds_tab(prmt(c, lane4, 0x7604u));
-                    pr[4 * i + 1] = lds_tab(prmt(c, lane4, 0x7614u));
-                    pr[4 * i + 2] = lds_tab(prmt(c, lane4, 0x7624u));
-                    pr[4 * i + 3] = lds_tab(prmt(c, lane4, 0x7634u));
-                }
             } else {
-                // one 12-byte group of 32 k: pair q (k 2q, 2q + 1) is the 6-bit field q % 5
-                // of word q / 5 (q < 15); pair 15 takes the two top bits of each word
-                // group gi's words are cw[4 gi .. 4 gi + 2] (its ring slot)
-                auto pair_off = [&](int q, int gi = 0) -> uint32_t {
-                    const uint32_t* g3 = cw + 4 * gi;
-                    if (q == 15)
-                        return ((g3[0] >> 22) & 0x0300u) | ((g3[1] >> 20) & 0x0c00u) | ((g3[2] >> 18) & 0x3000u) | lane4;
-                    const int f = q % 5;
-                    const uint32_t x = g3[q / 5];
-                    const uint32_t field = f == 0 ? (x << 8) : f == 1 ? (x << 2) : f == 2 ? (x >> 4)
-                                         : f == 3 ? (x >> 10) : (x >> 16);
-                    return (field & 0x3f00u) | lane4;
-                };
-                if constexpr (kSliceK == 64) {
-#pragma unroll
-                    for (int q = 0; q < 32; ++q) pr[q] = lds_tab(pair_off(q & 15, q >> 4));
-                } else if constexpr (kSliceK == 32) {
-#pragma unroll
-                    for (int q = 0; q < 16; ++q) pr[q] = lds_tab(pair_off(q));
+                uint32_t cw[4 * SLOTS];
+    #pragma unroll
+                for (int q = 0; q < SLOTS; ++q) {
+                    uint4 cv = make_uint4(0, 0, 0, 0);
+                    if (valid) cv = lds128(ring_slot(slot, SLOTS * d) + 16 * q);
+                    cw[4 * q] = cv.x; cw[4 * q + 1] = cv.y; cw[4 * q + 2] = cv.z; cw[4 * q + 3] = cv.w;
+                }
+                if (p.bits == 4) {
+                    // word i holds k = kSliceK h + 8i .. +7
+    #pragma unroll
+                    for (int i = 0; i < kSliceK / 8; ++i) {
+                        const uint32_t c = cw[i];
+                        pr[4 * i + 0] = lds_tab(prmt(c, lane4, 0x7604u));
+                        pr[4 * i + 1] = lds_tab(prmt(c, lane4, 0x7614u));
+                        pr[4 * i + 2] = lds_tab(prmt(c, lane4, 0x7624u));
+                        pr[4 * i + 3] = lds_tab(prmt(c, lane4, 0x7634u));
+                    }
                 } else {
-                    // this slice is half of the group: pairs 8 (h & 1) .. +7
-                    if ((h & 1) == 0) {
-#pragma unroll
-                        for (int q = 0; q < 8; ++q) pr[q] = lds_tab(pair_off(q));
+                    // one 12-byte group of 32 k: pair q (k 2q, 2q + 1) is the 6-bit field q % 5
+                    // of word q / 5 (q < 15); pair 15 takes the two top bits of each word
+                    // group gi's words are cw[4 gi .. 4 gi + 2] (its ring slot)
+                    auto pair_off = [&](int q, int gi = 0) -> uint32_t {
+                        const uint32_t* g3 = cw + 4 * gi;
+                        if (q == 15)
+                            return ((g3[0] >> 22) & 0x0300u) | ((g3[1] >> 20) & 0x0c00u) | ((g3[2] >> 18) & 0x3000u) | lane4;
+                        const int f = q % 5;
+                        const uint32_t x = g3[q / 5];
+                        const uint32_t field = f == 0 ? (x << 8) : f == 1 ? (x << 2) : f == 2 ? (x >> 4)
+                                             : f == 3 ? (x >> 10) : (x >> 16);
+                        return (field & 0x3f00u) | lane4;
+                    };
+                    if constexpr (kSliceK == 64) {
+    #pragma unroll
+                        for (int q = 0; q < 32; ++q) pr[q] = lds_tab(pair_off(q & 15, q >> 4));
+                    } else if constexpr (kSliceK == 32) {
+    #pragma unroll
+                        for (int q = 0; q < 16; ++q) pr[q] = lds_tab(pair_off(q));
                     } else {
-#pragma unroll
-                        for (int q = 0; q < 8; ++q) pr[q] = lds_tab(pair_off(8 + q));
+                        // this slice is half of the group: pairs 8 (h & 1) .. +7
+                        if ((h & 1) == 0) {
+    #pragma unroll
+                            for (int q = 0; q < 8; ++q) pr[q] = lds_tab(pair_off(q));
+                        } else {
+    #pragma unroll
+                            for (int q = 0; q < 8; ++q) pr[q] = lds_tab(pair_off(8 + q));
+                        }
                     }
                 }
             }
@@ -869,17 +892,30 @@ uint32_t make_idesc(bool f16_inputs, int bn)
 // Dynamic shared memory of the layout: table rows, X stages, barriers.
 constexpr uint32_t smem_bytes_for(int bn) { return kTabRegion + kXStages * (uint32_t)bn * kBK * 2 + 256; }
 
+// Outputs of a split launch: per matrix its partial sums [splits][count] and Y[count].
+struct SumArgs {
+    const float* part[kMaxPrefillItems];
+    void* Y[kMaxPrefillItems];
+    int64_t count[kMaxPrefillItems];        // B * N
+    int n;
+};
+
 // Fixed-order sum of the k ranges' fp32 partial sums: Y[i] = sum_s part[s][i]
-// (s = 0, 1, ...), rounded to Y's dtype.
-__global__ void __launch_bounds__(256) splitk_sum_kernel(const float* __restrict__ part, int splits, int64_t count,
-                                                         void* Y, int y_dtype)
+// (s = 0, 1, ...), rounded to Y's dtype, over the matrices of the launch in turn.
+__global__ void __launch_bounds__(256) splitk_sum_kernel(const __grid_constant__ SumArgs a, int splits, int64_t total,
+                                                         int y_dtype)
 {
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < count; i += (int64_t)gridDim.x * blockDim.x) {
+    for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < total; g += (int64_t)gridDim.x * blockDim.x) {
+        int m = 0;
+        int64_t i = g;
+        while (m + 1 < a.n && i >= a.count[m]) i -= a.count[m++];
+        const float* part = a.part[m];
+        const int64_t count = a.count[m];
         float v = part[i];
         for (int sp = 1; sp < splits; ++sp) v += part[(int64_t)sp * count + i];
-        if (y_dtype == LOGQ_F32) static_cast<float*>(Y)[i] = v;
-        else if (y_dtype == LOGQ_BF16) static_cast<__nv_bfloat16*>(Y)[i] = __float2bfloat16_rn(v);
-        else static_cast<__half*>(Y)[i] = __float2half_rn(v);
+        if (y_dtype == LOGQ_F32) static_cast<float*>(a.Y[m])[i] = v;
+        else if (y_dtype == LOGQ_BF16) static_cast<__nv_bfloat16*>(a.Y[m])[i] = __float2bfloat16_rn(v);
+        else static_cast<__half*>(a.Y[m])[i] = __float2half_rn(v);
     }
 }
 
@@ -909,13 +945,50 @@ cudaError_t launch(PrefillParams& p, const CUtensorMap& xmap, int grid, cudaStre
 
 }  // namespace
 
-PrefillPlan prefill_plan(int64_t B, int64_t N, int64_t K, size_t part_bytes_avail)
+PrefillPlan prefill_plan(int64_t B, const int64_t* N, int count, int64_t K, size_t part_bytes_avail)
 {
     PrefillPlan pl;
+    memset(&pl, 0, sizeof pl);
     pl.bn = B <= 16 ? 16 : kBNMax;
     const int sms = sm_count() > 0 ? sm_count() : 148;
-    const int64_t tiles = ((N + kBM - 1) / kBM) * ((B + pl.bn - 1) / pl.bn);
+    const int64_t ttiles = (B + pl.bn - 1) / pl.bn;
+    int64_t tiles[kMaxPrefillItems], sum_n = 0;
+    for (int i = 0; i < count; ++i) {
+        tiles[i] = ((N[i] + kBM - 1) / kBM) * ttiles;
+        sum_n += N[i];
+    }
     const int64_t ksteps = K / kBK;
+    // CTAs per matrix for `splits` k ranges per tile: a share of the grid in
+    // proportion to the matrix's work units, then each CTA left over to the
+    // matrix whose CTAs take the most rounds.  Returns those rounds.
+    auto share = [&](int64_t splits, int* ncta) -> int64_t {
+        int64_t units[kMaxPrefillItems], total = 0;
+        for (int i = 0; i < count; ++i) total += (units[i] = tiles[i] * splits);
+        const int64_t grid = total < sms ? total : sms;
+        int64_t used = 0;
+        for (int i = 0; i < count; ++i) {
+            int64_t c = grid * units[i] / total;
+            c = c < 1 ? 1 : (c > units[i] ? units[i] : c);
+            ncta[i] = (int)c;
+            used += c;
+        }
+        auto rounds = [&](int i) { return (units[i] + ncta[i] - 1) / ncta[i]; };
+        while (used < grid) {
+            int best = -1;
+            for (int i = 0; i < count; ++i) {
+                if (ncta[i] >= units[i]) continue;
+                if (best < 0 || rounds(i) > rounds(best) ||
+                    (rounds(i) == rounds(best) && units[i] * ncta[best] > units[best] * ncta[i]))
+                    best = i;
+            }
+            if (best < 0) break;
+            ++ncta[best];
+            ++used;
+        }
+        int64_t r = 0;
+        for (int i = 0; i < count; ++i) r = rounds(i) > r ? rounds(i) : r;
+        return r;
+    };
     // Cost in k-step times (~0.5 us each on the GB300, for either tile width;
     // the decode warps bound a stage): persistent CTAs take tiles in rounds,
     // a tile of ks k-steps costing ks + 6 (pipeline fill, and the MMA waiting
@@ -924,10 +997,10 @@ PrefillPlan prefill_plan(int64_t B, int64_t N, int64_t K, size_t part_bytes_avai
     // (8 bytes per output and range, at ~6 TB/s).  Each range keeps at least 8
     // k-steps and the partials fit the caller's workspace.  (Fitted to launches
     // of the Llama-3.1-8B shapes at batches 8-64 and 2048 tokens.)
+    int ncta[kMaxPrefillItems];
     auto cost = [&](int64_t splits, int64_t ksplit) {
-        const int64_t units = tiles * splits;
-        double c = (double)((units + sms - 1) / sms) * (double)(ksplit + 6);
-        if (splits > 1) c += 6.0 + (double)splits * (double)B * (double)N * 8.0 / 3.0e6;
+        double c = (double)share(splits, ncta) * (double)(ksplit + 6);
+        if (splits > 1) c += 6.0 + (double)splits * (double)B * (double)sum_n * 8.0 / 3.0e6;
         return c;
     };
     pl.splits = 1;
@@ -936,7 +1009,7 @@ PrefillPlan prefill_plan(int64_t B, int64_t N, int64_t K, size_t part_bytes_avai
     for (int64_t sp = 2; sp <= 32 && ksteps / sp >= 8; ++sp) {
         const int64_t ksplit = (ksteps + sp - 1) / sp;
         const int64_t real = (ksteps + ksplit - 1) / ksplit;       // ranges actually used
-        const size_t need = (size_t)real * (size_t)B * (size_t)N * 4;
+        const size_t need = (size_t)real * (size_t)B * (size_t)sum_n * 4;
         if (need > part_bytes_avail) break;
         const double c = cost(real, ksplit);
         if (c < best) {
@@ -945,62 +1018,110 @@ PrefillPlan prefill_plan(int64_t B, int64_t N, int64_t K, size_t part_bytes_avai
             pl.ksplit = (int)ksplit;
         }
     }
-    pl.part_bytes = pl.splits > 1 ? (size_t)pl.splits * (size_t)B * (size_t)N * 4 : 0;
+    share(pl.splits, pl.ncta);
+    pl.part_bytes = pl.splits > 1 ? (size_t)pl.splits * (size_t)B * (size_t)sum_n * 4 : 0;
     pl.est_us = 0.5 * best + 3.0;
     return pl;
 }
 
-cudaError_t launch_prefill(const LinearArgs& a, cudaStream_t s)
+PrefillPlan prefill_plan(int64_t B, int64_t N, int64_t K, size_t part_bytes_avail)
+{
+    return prefill_plan(B, &N, 1, K, part_bytes_avail);
+}
+
+namespace {
+
+// One launch over `count` matrices that share X (and the split k ranges'
+// sum kernel where the plan splits them).
+cudaError_t launch_items(const GroupItem* gi, int count, const void* X, int x_f16, int64_t B, int64_t K, int bits,
+                         int y_dtype, Workspace* ws, size_t ws_bytes, cudaStream_t s)
 {
     auto encode = encode_fn();
     if (!encode) return cudaErrorNotSupported;
+    int64_t Ns[kMaxPrefillItems];
+    for (int i = 0; i < count; ++i) Ns[i] = gi[i].N;
+    const size_t avail = ws_bytes > kWorkspaceBytes ? ws_bytes - kWorkspaceBytes : 0;
+    const PrefillPlan pl = prefill_plan(B, Ns, count, K, avail);
     CUtensorMap xmap;
     memset(&xmap, 0, sizeof xmap);
-    const cuuint64_t gdim[2] = {(cuuint64_t)a.K, (cuuint64_t)a.B};
-    const cuuint64_t gstride[1] = {(cuuint64_t)a.K * 2};
-    const size_t avail = a.ws_bytes > kWorkspaceBytes ? a.ws_bytes - kWorkspaceBytes : 0;
-    const PrefillPlan pl = prefill_plan(a.B, a.N, a.K, avail);
+    const cuuint64_t gdim[2] = {(cuuint64_t)K, (cuuint64_t)B};
+    const cuuint64_t gstride[1] = {(cuuint64_t)K * 2};
     const cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)pl.bn};
     const cuuint32_t estride[2] = {1, 1};
-    CUresult r = encode(&xmap, a.x_f16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
-                        const_cast<void*>(a.X), gdim, gstride, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
+    CUresult r = encode(&xmap, x_f16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                        const_cast<void*>(X), gdim, gstride, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
                         CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
 
     PrefillParams p;
     memset(&p, 0, sizeof p);
-    p.codes = a.codes;
-    p.Y = a.Y;
-    p.ws = a.ws;
-    p.N = a.N;
-    p.K = (int32_t)a.K;
-    p.B = (int32_t)a.B;
-    p.bits = a.bits;
-    p.row_bytes = (a.bits == 8) ? a.K : (a.bits == 4) ? a.K / 2 : a.K / 32 * 12;
-    p.y_dtype = a.y_dtype;
-    p.n_tiles_n = (int32_t)((a.N + kBM - 1) / kBM);
-    p.n_tiles_t = (int32_t)((a.B + pl.bn - 1) / pl.bn);
+    p.nitems = count;
+    p.ws = ws;
+    p.K = (int32_t)K;
+    p.B = (int32_t)B;
+    p.bits = bits;
+    p.row_bytes = (bits == 8) ? K : (bits == 4) ? K / 2 : K / 32 * 12;
+    p.y_dtype = y_dtype;
+    p.n_tiles_t = (int32_t)((B + pl.bn - 1) / pl.bn);
     p.splits = pl.splits;
     p.ksplit = pl.ksplit;
-    p.part = pl.splits > 1 ? reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(a.ws) + kWorkspaceBytes) : nullptr;
-    p.idesc = make_idesc(a.x_f16 != 0, pl.bn);
-    for (int c = 0; c < (1 << a.bits); ++c) p.lvl16[c] = a.lvl16[c];
-    const int64_t ntiles = (int64_t)p.n_tiles_n * p.n_tiles_t * p.splits;
-    const int sms = sm_count() > 0 ? sm_count() : 148;
-    const int grid = (int)(ntiles < sms ? ntiles : sms);
+    p.idesc = make_idesc(x_f16 != 0, pl.bn);
+    // partial sums of matrix i after those of matrices 0 .. i-1
+    float* part = pl.splits > 1 ? reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(ws) + kWorkspaceBytes) : nullptr;
+    SumArgs sa;
+    memset(&sa, 0, sizeof sa);
+    sa.n = count;
+    int grid = 0;
+    int64_t total = 0;
+    for (int i = 0; i < count; ++i) {
+        PrefillItem& it = p.item[i];
+        it.codes = gi[i].codes;
+        it.Y = gi[i].Y;
+        it.N = gi[i].N;
+        it.n_tiles_n = (int32_t)((gi[i].N + kBM - 1) / kBM);
+        it.cta_begin = grid;
+        it.ncta = pl.ncta[i];
+        it.part = part;
+        for (int c = 0; c < (1 << bits); ++c) it.lvl16[c] = gi[i].lvl16[c];
+        grid += pl.ncta[i];
+        sa.part[i] = part;
+        sa.Y[i] = gi[i].Y;
+        sa.count[i] = B * gi[i].N;
+        total += B * gi[i].N;
+        if (part) part += (int64_t)pl.splits * B * gi[i].N;
+    }
 
     cudaError_t e;
     if (pl.bn == 16)
-        e = a.bits == 8 ? launch<true, 16>(p, xmap, grid, s) : launch<false, 16>(p, xmap, grid, s);
+        e = bits == 8 ? launch<true, 16>(p, xmap, grid, s) : launch<false, 16>(p, xmap, grid, s);
     else
-        e = a.bits == 8 ? launch<true, kBNMax>(p, xmap, grid, s) : launch<false, kBNMax>(p, xmap, grid, s);
+        e = bits == 8 ? launch<true, kBNMax>(p, xmap, grid, s) : launch<false, kBNMax>(p, xmap, grid, s);
     if (e != cudaSuccess || pl.splits == 1) return e;
-    const int64_t count = a.B * a.N;
-    int64_t blocks = (count + 255) / 256;
+    const int sms = sm_count() > 0 ? sm_count() : 148;
+    int64_t blocks = (total + 255) / 256;
     if (blocks > (int64_t)sms * 8) blocks = (int64_t)sms * 8;
-    splitk_sum_kernel<<<(int)blocks, 256, 0, s>>>(p.part, pl.splits, count, a.Y, a.y_dtype);
+    splitk_sum_kernel<<<(int)blocks, 256, 0, s>>>(sa, pl.splits, total, y_dtype);
     return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_prefill(const LinearArgs& a, cudaStream_t s)
+{
+    GroupItem gi;
+    memset(&gi, 0, sizeof gi);
+    gi.codes = a.codes;
+    gi.Y = a.Y;
+    gi.N = a.N;
+    for (int c = 0; c < (1 << a.bits); ++c) gi.lvl16[c] = a.lvl16[c];
+    return launch_items(&gi, 1, a.X, a.x_f16, a.B, a.K, a.bits, a.y_dtype, a.ws, a.ws_bytes, s);
+}
+
+cudaError_t launch_prefill_group(const GroupArgs& g, size_t ws_bytes, cudaStream_t s)
+{
+    if (g.count < 1 || g.count > kMaxPrefillItems) return cudaErrorInvalidValue;
+    return launch_items(g.item, g.count, g.X, g.x_f16, g.B, g.K, g.bits, g.y_dtype, g.ws, ws_bytes, s);
 }
 
 }  // namespace logq

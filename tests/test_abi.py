@@ -114,6 +114,25 @@ def test_linear_workspace_bytes(logq):
     assert logq.logq_linear_workspace_bytes(16, 4096, 100, 4) == 0
 
 
+def test_linear_grouped_workspace_bytes(logq):
+    """A group that runs as one tensor-core launch asks for the partial sums of all its
+    matrices (splits x B x sum(N) fp32), one that runs on the CUDA cores or unsplit only
+    for the base workspace; a single matrix asks what logq_linear asks; invalid groups
+    give 0."""
+    base = logq.logq_workspace_bytes()
+    g = logq.logq_linear_grouped_workspace_bytes
+    assert g(64, [1024, 512, 512], 4096, 4) == base + 8 * 64 * 2048 * 4
+    assert g(2048, [4096, 1024, 1024], 4096, 4) == base        # one unsplit launch fills the GPU
+    assert g(4, [4096, 1024, 1024], 4096, 4) == base
+    assert g(1, [14336, 14336], 4096, 4) == base
+    for B, N, K, bits in [(16, 4096, 8192, 4), (64, 1024, 4096, 4), (2048, 1024, 4096, 4), (1, 4096, 4096, 4)]:
+        assert g(B, [N], K, bits) == logq.logq_linear_workspace_bytes(B, N, K, bits)
+    assert g(64, [], 4096, 4) == 0
+    assert g(64, [64] * 5, 4096, 4) == 0
+    assert g(64, [64, 64], 100, 4) == 0
+    assert g(0, [64], 4096, 4) == 0
+
+
 def test_status_strings(logq):
     for s in range(7):
         assert len(logq.status_string(s)) >= 2

@@ -217,15 +217,17 @@ def test_prefill_split_k_dtypes(logq, bits, N, K, B, xdt):
 
 
 def test_grouped_split_k_equals_single_calls(logq):
-    """A grouped call at batch 64 runs each matrix on the tensor cores with its k range
-    split, one after another through the same workspace: each output equals the single
-    call's bit for bit and matches the oracle."""
+    """A grouped call at batch 64 runs its three matrices in one tensor-core launch with
+    every k range split in eight (the partial sums of each matrix after the previous
+    one's in the workspace), as each single call splits its own: each output equals the
+    single call's bit for bit and matches the oracle."""
     K, B = 4096, 64
     shapes = [(1024, 1.4), (512, 1.7), (512, 2.0)]
     layers = [make_layer(logq, N, K, 4, base, seed=90 + i) for i, (N, base) in enumerate(shapes)]
     X = workloads.activations_torch(B, K, 91, torch.bfloat16, "cuda")
-    wsb = max(logq.logq_linear_workspace_bytes(B, N, K, 4) for N, _ in shapes)
-    assert wsb > logq.logq_workspace_bytes()
+    wsb = logq.logq_linear_grouped_workspace_bytes(B, [N for N, _ in shapes], K, 4)
+    # one launch: partial sums of all three matrices, 8 ranges each
+    assert wsb == logq.logq_workspace_bytes() + 8 * B * sum(N for N, _ in shapes) * 4
     ws = logq.new_workspace(nbytes=wsb)
     items = [(codes, cb, N, None) for (codes, cb, ocb, q), (N, _) in zip(layers, shapes)]
     outs = logq.logq_linear_grouped(items, X, K, y_dtype=torch.bfloat16, workspace=ws)
@@ -233,6 +235,37 @@ def test_grouped_split_k_equals_single_calls(logq):
         assert torch.equal(Y, logq.logq_linear(codes, cb, X, N, K, y_dtype=torch.bfloat16, workspace=ws))
         Yr, A = reference(X, q, ocb)
         check_linear(Y.double().cpu().numpy(), Yr, A, "bf16")
+    st, detail = logq.logq_workspace_status(ws)
+    assert st == logq.LOGQ_OK and detail == 0
+
+
+@pytest.mark.parametrize("bits,B,shapes,K", [
+    (4, 300, [(2000, 1.4), (500, 1.7), (520, 2.0)], 1024),      # q/k/v-like, ragged rows and tokens
+    (4, 512, [(2048, 1.3), (512, 1.6)], 1024),
+    (3, 96, [(640, 1.25), (256, 1.4)], 1152),
+    (8, 200, [(384, 1.05), (136, 1.02), (64, 1.03), (256, 1.04)], 512),
+    (4, 12, [(8192, 1.5), (8192, 1.8)], 4096),                   # gate/up-like, 16-token tiles
+])
+def test_grouped_tensor_core_launch(logq, bits, B, shapes, K):
+    """Matrices sharing X in one tensor-core launch (each a share of the CTAs, its own
+    table): every output matches the oracle, with and without room for split k ranges.
+    Unsplit, above batch 16 (where a single call also runs on the tensor cores), each
+    equals the single call's bit for bit (same tiles, same k order)."""
+    layers = [make_layer(logq, N, K, bits, base, seed=110 + i) for i, (N, base) in enumerate(shapes)]
+    X = workloads.activations_torch(B, K, 111, torch.bfloat16, "cuda")
+    items = [(codes, cb, N, None) for (codes, cb, ocb, q), (N, _) in zip(layers, shapes)]
+    outs = logq.logq_linear_grouped(items, X, K, y_dtype=torch.bfloat16)
+    for (codes, cb, ocb, q), Y in zip(layers, outs):
+        Yr, A = reference(X, q, ocb)
+        check_linear(Y.double().cpu().numpy(), Yr, A, "bf16")
+    ws = logq.new_workspace()
+    outs1 = logq.logq_linear_grouped(items, X, K, y_dtype=torch.bfloat16, workspace=ws)
+    for (codes, cb, ocb, q), (N, _), Y in zip(layers, shapes, outs1):
+        if B > 16:
+            assert torch.equal(Y, logq.logq_linear(codes, cb, X, N, K, y_dtype=torch.bfloat16, workspace=ws))
+        else:
+            Yr, A = reference(X, q, ocb)
+            check_linear(Y.double().cpu().numpy(), Yr, A, "bf16")
     st, detail = logq.logq_workspace_status(ws)
     assert st == logq.LOGQ_OK and detail == 0
 
