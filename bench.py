@@ -461,48 +461,86 @@ def time_gptq(logq, torch, dev):
 
 
 def time_prefill(logq, torch, dev, reps: int = 3):
-    """Prefill GEMM: 2048 tokens x each Llama-3.1-8B linear shape."""
-    res = {}
-    # room for split-k partial sums of every shape (k/v: too few output tiles to fill the GPU)
-    ws = logq.new_workspace(dev, max(logq.logq_linear_workspace_bytes(PREFILL_TOKENS, N, K, 4)
-                                     for N, K in workloads.LLAMA_8B_SHAPES.values()))
+    """Prefill GEMM at 2048 tokens on one Llama-3.1-8B layer's linears: each shape in a
+    launch of its own, and the layer as a model runs it -- q/k/v in one grouped launch
+    (they read the same X), o, gate/up in one grouped launch, down."""
+    sh = workloads.LLAMA_8B_SHAPES
+    T = PREFILL_TOKENS
+    groups = {"qkv": ("q", "k", "v"), "gateup": ("gate", "up")}
+    # room for split-k partial sums of every launch (k/v alone: too few output tiles)
+    wsb = max([logq.logq_linear_workspace_bytes(T, N, K, 4) for N, K in sh.values()] +
+              [logq.logq_linear_grouped_workspace_bytes(T, [sh[n][0] for n in g], sh[g[0]][1], 4)
+               for g in groups.values()])
+    ws = logq.new_workspace(dev, wsb)
     s = torch.cuda.Stream(dev)
-    tot_flop, tot_t = 0.0, 0.0
+    mats = {}
     for pi, name in enumerate(workloads.PROJ_NAMES):
-        if name in ("v", "up"):
-            continue                                 # same shapes as k and gate
-        N, K = workloads.LLAMA_8B_SHAPES[name]
+        N, K = sh[name]
         W = workloads.weights_torch(N, K, workloads.layer_seed(4, 0, pi), outliers=True, device=dev)
         codes, cb = logq.logq_quantize(W, 4, 1.5, workspace=ws)
         del W
-        X = workloads.activations_torch(PREFILL_TOKENS, K, pi, torch.bfloat16, dev)
-        Y = torch.empty(PREFILL_TOKENS, N, dtype=torch.bfloat16, device=dev)
-        try:
-            logq.logq_linear(codes, cb, X, N, K, y_dtype=torch.bfloat16, Y=Y, workspace=ws, stream=s)
-        except logq.LogqError as e:
-            if e.status == logq.LOGQ_ERR_UNSUPPORTED:
-                return None
-            raise
-        torch.cuda.synchronize()
+        mats[name] = (codes, cb, N, K, torch.empty(T, N, dtype=torch.bfloat16, device=dev))
+    xs = {K: workloads.activations_torch(T, K, K, torch.bfloat16, dev) for K in {k for _, k in sh.values()}}
+
+    def single(name):
+        codes, cb, N, K, Y = mats[name]
+        logq.logq_linear(codes, cb, xs[K], N, K, y_dtype=torch.bfloat16, Y=Y, workspace=ws, stream=s)
+
+    def grouped(key):
+        names = groups[key]
+        K = mats[names[0]][3]
+        logq.logq_linear_grouped([(mats[n][0], mats[n][1], mats[n][2], mats[n][4]) for n in names], xs[K], K,
+                                 y_dtype=torch.bfloat16, workspace=ws, stream=s)
+
+    def timed(fn):
         # reps back-to-back calls captured in a graph (a split call is two launches:
         # the GEMM and the sum of its k ranges), so host launch gaps stay out
+        fn()
+        torch.cuda.synchronize()
         g = torch.cuda.CUDAGraph()
         with torch.cuda.stream(s):
             with torch.cuda.graph(g, stream=s):
                 for _ in range(reps):
-                    logq.logq_linear(codes, cb, X, N, K, y_dtype=torch.bfloat16, Y=Y, workspace=ws, stream=s)
+                    fn()
         g.replay()
         torch.cuda.synchronize()
         t = time_replays(torch, g, s, 2) / (2 * reps)
         del g
-        flop = 2.0 * PREFILL_TOKENS * N * K
-        res[name] = {"N": N, "K": K, "us": round(t * 1e6, 2), "tflops": round(flop / t / 1e12, 1)}
-        tot_flop += flop * (2 if name in ("k", "gate") else 1)
-        tot_t += t * (2 if name in ("k", "gate") else 1)
-        del codes, X, Y
+        return t
+
+    try:
+        single("q")
+    except logq.LogqError as e:
+        if e.status == logq.LOGQ_ERR_UNSUPPORTED:
+            return None
+        raise
+    res, grp = {}, {}
+    one_flop, one_t = 0.0, 0.0
+    for name in workloads.PROJ_NAMES:
+        N, K = sh[name]
+        flop = 2.0 * T * N * K
+        if name in ("v", "up"):                      # same shapes as k and gate
+            t = res["k" if name == "v" else "gate"]["us"] * 1e-6
+        else:
+            t = timed(lambda: single(name))
+            res[name] = {"N": N, "K": K, "us": round(t * 1e6, 2), "tflops": round(flop / t / 1e12, 1)}
+        one_flop += flop
+        one_t += t
+    layer_flop, layer_t = 0.0, 0.0
+    for key, names in groups.items():
+        t = timed(lambda: grouped(key))
+        flop = sum(2.0 * T * sh[n][0] * sh[n][1] for n in names)
+        grp[key] = {"N": sum(sh[n][0] for n in names), "K": sh[names[0]][1], "us": round(t * 1e6, 2),
+                    "tflops": round(flop / t / 1e12, 1)}
+        layer_flop += flop
+        layer_t += t
+    for name in ("o", "down"):
+        layer_flop += 2.0 * T * sh[name][0] * sh[name][1]
+        layer_t += res[name]["us"] * 1e-6
     st, _ = logq.logq_workspace_status(ws)
     assert st == logq.LOGQ_OK, "prefill pipeline reported a timeout"
-    return {"layers": res, "tflops": tot_flop / tot_t / 1e12}
+    return {"layers": res, "grouped": grp, "tflops": layer_flop / layer_t / 1e12,
+            "tflops_one_launch_per_matrix": one_flop / one_t / 1e12, "layer_us": round(layer_t * 1e6, 1)}
 
 
 def replica_totals(t_local: float, units_local: float, dist=None, device=None):
@@ -814,7 +852,12 @@ def run_ours(args):
                 line["prefill"] = {"tflops": round(pf["tflops"], 1), "unit": "TFLOP/s",
                                    "peak": pk["bf16_tflops"],
                                    "frac": round(pf["tflops"] / pk["bf16_tflops"], 4),
-                                   "layers": pf["layers"], "tokens": PREFILL_TOKENS}
+                                   "layer_us": pf["layer_us"], "grouped": pf["grouped"],
+                                   "layers": pf["layers"], "tokens": PREFILL_TOKENS,
+                                   "tflops_one_launch_per_matrix": round(pf["tflops_one_launch_per_matrix"], 1),
+                                   "note": "tflops: one Llama-3.1-8B layer's linears as a model runs them "
+                                           "(q/k/v one grouped launch, o, gate/up one grouped launch, down); "
+                                           "layers: each shape in a launch of its own"}
             else:
                 line["prefill"] = None
         except Exception as e:
@@ -827,14 +870,15 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
-CASES = ("decode_layers_8b", "decode_step_1b", "skinny_gate_8b", "gemv_gateup_1b", "gemv_gate_8b", "prefill_q_8b", "quantize_gate_8b", "energy_gate_8b",
+CASES = ("decode_layers_8b", "decode_step_1b", "skinny_gate_8b", "gemv_gateup_1b", "gemv_gate_8b", "prefill_q_8b",
+         "prefill_qkv_8b", "quantize_gate_8b", "energy_gate_8b",
          "gemv8_gate_8b", "gptq_q_8b", "gptq_update_q_8b", "quantize3_gate_8b")
 
 
 def run_case(name: str):
     """One small workload run twice (for a profiler capture of the second run):
     the gate+up launch of the 1B decode step, the 8B gate GEMV, the 8B q-shaped
-    prefill GEMM (2048 tokens), the quantisation of an 8B gate matrix, its
+    prefill GEMM (2048 tokens) and the grouped q/k/v one, the quantisation of an 8B gate matrix, its
     self-calibrating (energy-range) quantisation, the 8-bit gate GEMV and 4-bit
     GPTQ of an 8B q matrix (factor and quantisation; or the quantisation alone with a
     fixed upper-triangular factor standing in for U)."""
@@ -884,6 +928,16 @@ def run_case(name: str):
         X = workloads.activations_torch(PREFILL_TOKENS, K, 2, torch.bfloat16, dev)
         for _ in range(2):
             logq.logq_linear(c[0], c[1], X, N, K, y_dtype=torch.bfloat16, workspace=ws)
+    elif name == "prefill_qkv_8b":
+        K = workloads.LLAMA_8B_SHAPES["q"][1]
+        items = []
+        for i, proj in enumerate(("q", "k", "v")):
+            N = workloads.LLAMA_8B_SHAPES[proj][0]
+            c = logq.logq_quantize(workloads.weights_torch(N, K, 20 + i, True, dev), 4, 1.5, workspace=ws)
+            items.append((c[0], c[1], N, None))
+        X = workloads.activations_torch(PREFILL_TOKENS, K, 2, torch.bfloat16, dev)
+        for _ in range(2):
+            logq.logq_linear_grouped(items, X, K, y_dtype=torch.bfloat16, workspace=ws)
     elif name == "quantize_gate_8b":
         N, K = workloads.LLAMA_8B_SHAPES["gate"]
         W = workloads.weights_torch(N, K, 15, True, dev)
