@@ -201,9 +201,9 @@ logq_status logq_linear(const uint8_t* codes, const logq_codebook* cb, const voi
  * or other allocating routine.  Its first call on a device (and the first call
  * after the device's context has been replaced, e.g. by cudaDeviceReset) looks
  * up the array's device address with that device current.  All calls share
- * the one array, which
- * keeps the last call's contents (each call clears the words it needs): calls
- * that overlap on the GPU race and must be serialised by the caller.  Like
+ * the one array, which keeps the last call's contents (each call clears the
+ * words it needs): calls that overlap on the GPU race and must be serialised
+ * by the caller.  Like
  * logq_quantize it synchronises `stream` before returning; arguments and
  * errors are those of logq_quantize, and the quantisation is the same code.
  */
