@@ -958,17 +958,18 @@ PrefillPlan prefill_plan(int64_t B, const int64_t* N, int count, int64_t K, size
         sum_n += N[i];
     }
     const int64_t ksteps = K / kBK;
-    // CTAs per matrix for `splits` k ranges per tile: a share of the grid in
-    // proportion to the matrix's work units, then each CTA left over to the
-    // matrix whose CTAs take the most rounds.  Returns those rounds.
+    // CTAs per matrix for `splits` k ranges per tile: one each, a share of the
+    // rest of the grid in proportion to the matrix's work units, then each CTA
+    // left over to the matrix whose CTAs take the most rounds (the grid never
+    // exceeds the SMs).  Returns those rounds.
     auto share = [&](int64_t splits, int* ncta) -> int64_t {
         int64_t units[kMaxPrefillItems], total = 0;
         for (int i = 0; i < count; ++i) total += (units[i] = tiles[i] * splits);
         const int64_t grid = total < sms ? total : sms;
         int64_t used = 0;
         for (int i = 0; i < count; ++i) {
-            int64_t c = grid * units[i] / total;
-            c = c < 1 ? 1 : (c > units[i] ? units[i] : c);
+            int64_t c = 1 + (grid - count) * units[i] / total;
+            c = c > units[i] ? units[i] : c;
             ncta[i] = (int)c;
             used += c;
         }
