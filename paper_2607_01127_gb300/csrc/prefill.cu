@@ -7,7 +7,10 @@
 // = 256 for prefill and 16 for small batches; where there are too few tiles
 // to fill the SMs, each tile's k range is split into ranges taken by
 // different CTAs, which write fp32 partial sums to the caller's workspace and
-// a second kernel adds them in a fixed order.
+// a second kernel adds them in a fixed order.  A launch may cover up to four
+// matrices that read the same X (q/k/v, gate/up): each gets a contiguous
+// range of the CTAs, in proportion to its tiles, and a CTA works on its
+// matrix's tiles only.
 // The dequantised weight tile (the MMA's A operand) lives in tensor memory, not
 // in shared memory: tensor memory holds one fp32 accumulator (256 columns) and
 // eight weight stages (32 columns each), and shared memory holds the pair table
