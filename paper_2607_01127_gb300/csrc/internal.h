@@ -57,8 +57,8 @@ struct LinearArgs {
     size_t ws_bytes;        // the caller's workspace bytes (beyond kWorkspaceBytes: split-k partial sums)
 };
 
-// A grouped decode launch: up to four matrices that share X (e.g. q/k/v or
-// gate/up), each with its own codebook and output.
+// A grouped launch (decode GEMV or tensor-core prefill): up to four matrices
+// that share X (e.g. q/k/v or gate/up), each with its own codebook and output.
 struct GroupItem {
     const uint8_t* codes;
     void* Y;
