@@ -125,6 +125,11 @@ def test_linear_grouped_workspace_bytes(logq):
     assert g(2048, [4096, 1024, 1024], 4096, 4) == base        # one unsplit launch fills the GPU
     assert g(4, [4096, 1024, 1024], 4096, 4) == base
     assert g(1, [14336, 14336], 4096, 4) == base
+    # 3-bit group at batch 96: one launch, every k range split in two
+    assert g(96, [640, 256], 1152, 3) == base + 2 * 96 * 896 * 4
+    # q/k/v at batch 16: the tensor-core group with k split in three beats the
+    # CUDA-core group launch and the single calls
+    assert g(16, [4096, 1024, 1024], 4096, 4) == base + 3 * 16 * 6144 * 4
     for B, N, K, bits in [(16, 4096, 8192, 4), (64, 1024, 4096, 4), (2048, 1024, 4096, 4), (1, 4096, 4096, 4)]:
         assert g(B, [N], K, bits) == logq.logq_linear_workspace_bytes(B, N, K, bits)
     assert g(64, [], 4096, 4) == 0
