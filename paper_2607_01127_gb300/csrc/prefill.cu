@@ -993,8 +993,9 @@ PrefillPlan prefill_plan(int64_t B, const int64_t* N, int count, int64_t K, size
         for (int i = 0; i < count; ++i) r = rounds(i) > r ? rounds(i) : r;
         return r;
     };
-    // Cost in k-step times (~0.5 us each on the GB300, for either tile width;
-    // the decode warps bound a stage): persistent CTAs take tiles in rounds,
+    // Cost in k-step times (~0.5 us each on the GB300, for either tile width:
+    // the roles' hand-offs and the decode threads' code copies, more than the
+    // MMAs, set a stage's time): persistent CTAs take tiles in rounds,
     // a tile of ks k-steps costing ks + 6 (pipeline fill, and the MMA waiting
     // for the epilogue to drain the single accumulator).  A split adds the sum
     // kernel (~6) and the partial sums' HBM traffic, written once and read once
